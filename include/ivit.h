@@ -1,0 +1,145 @@
+/*
+ * ivit -- incremental ViT encoding of streaming camera frames on one GB300 (sm_103a).
+ *
+ * The library implements temporal token reuse (Sec. III-B of "Reducing Temporal
+ * Redundancy for Efficient Vision-Language-Action Inference"): a frame is encoded
+ * in full once (the paper's "odd chunk"); every later frame re-encodes only the
+ * tokens whose patch embedding changed (Eq. 3 score, threshold or top-k selection),
+ * with their queries attending over all tokens and the other tokens' per-layer K/V
+ * read from a resident cache (Eq. 4-5); reused tokens keep their cached outputs.
+ *
+ * Conventions for every entry point:
+ *  - Return value: IVIT_OK (0) or a negative IVIT_ERR_* code.  Nothing throws or
+ *    aborts across the ABI; ivit_last_error() describes the last failure.
+ *  - Device pointers ("_dev") are caller-owned CUDA global memory on the device the
+ *    handle was created on; host pointers ("_host") are caller-owned host memory.
+ *    The library never frees caller memory.  All work is enqueued on the caller's
+ *    cudaStream_t (passed as void*, NULL = legacy default stream) and is
+ *    asynchronous: outputs are valid once that stream has reached the call.
+ *  - A handle owns the weights (copied at create), every per-view cache and all
+ *    workspaces.  One handle may be used from one host thread at a time; calls on
+ *    one handle must be ordered on one stream (or explicitly synchronised).
+ *  - Shapes: S = n_streams camera streams, V = n_views views each, SV = S*V
+ *    independent views (each with its own caches), N = (img_h/patch)*(img_w/patch)
+ *    tokens per view, D = dim, L = depth, F = mlp_dim.
+ */
+#ifndef IVIT_H
+#define IVIT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define IVIT_OK 0
+#define IVIT_ERR_ARG (-1)      /* null handle/pointer, bad enum, out-of-range index */
+#define IVIT_ERR_SHAPE (-2)    /* configuration the kernels do not support */
+#define IVIT_ERR_OOM (-3)      /* device allocation failed */
+#define IVIT_ERR_CUDA (-4)     /* a CUDA runtime/driver call failed */
+#define IVIT_ERR_DEVICE (-5)   /* a kernel reported an error (bounded wait expired) */
+
+#define IVIT_GELU_TANH 0       /* 0.5x(1+tanh(sqrt(2/pi)(x+0.044715x^3))) (SigLIP) */
+#define IVIT_GELU_ERF 1        /* 0.5x(1+erf(x/sqrt 2)) (ViT) */
+#define IVIT_SEL_THRESHOLD 0   /* update token i iff sim(i) < threshold (strict) */
+#define IVIT_SEL_TOPK 1        /* update the topk lowest sims, ties by lower index */
+#define IVIT_REF_PREV_FRAME 0  /* reference = previous frame's embeddings (all tokens) */
+#define IVIT_REF_LAST_REFRESH 1 /* reference of token i updated only when i is updated */
+
+/* Encoder + selection configuration.
+ * Supported by the kernels: patch >= 1 dividing img_h and img_w; N <= 1024;
+ * dim % 64 == 0 and heads dividing dim with head_dim = dim/heads a multiple of 8,
+ * at most 128; mlp_dim % 8 == 0; SV <= 4096. */
+typedef struct ivit_config {
+  int32_t img_h, img_w;  /* frame size in pixels */
+  int32_t patch;         /* patch edge P; patch k-vector is P*P*3 (HWC order) */
+  int32_t dim;           /* D */
+  int32_t depth;         /* L transformer blocks (pre-LN) */
+  int32_t heads;         /* H */
+  int32_t mlp_dim;       /* F */
+  int32_t n_streams;     /* S */
+  int32_t n_views;       /* V */
+  float ln_eps;          /* layer-norm epsilon (1e-6) */
+  int32_t gelu;          /* IVIT_GELU_* */
+  int32_t select_mode;   /* IVIT_SEL_* */
+  float threshold;       /* IVIT_SEL_THRESHOLD: refresh where sim < threshold */
+  int32_t topk;          /* IVIT_SEL_TOPK: tokens refreshed per view, clamped to [0, N] */
+  int32_t ref_mode;      /* IVIT_REF_* */
+} ivit_config;
+
+typedef struct ivit_handle ivit_handle;
+
+/* Number of bf16 elements of the weight buffer for `cfg`, 0 if cfg is invalid.
+ * Layout (row-major tensors, back to back):
+ *   W_pe[D][P*P*3] (column k = (ky*P+kx)*3+c, applied to pixel-128), b_pe[D], pos[N][D],
+ *   per layer: ln1_g[D] ln1_b[D] W_qkv[3D][D] b_qkv[3D] W_o[D][D] b_o[D]
+ *              ln2_g[D] ln2_b[D] W_1[F][D] b_1[F] W_2[D][F] b_2[D],
+ *   lnf_g[D] lnf_b[D].
+ * W_qkv rows: query block, key block, value block; head h owns rows h*dh..h*dh+dh-1
+ * of each block (Eq. 4: Q = W_Q T, K = W_K T, V = W_V T). */
+size_t ivit_weights_size(const ivit_config* cfg);
+
+/* Creates a handle on the current CUDA device: validates cfg, copies the weights
+ * (bf16 bit patterns, host memory, ivit_weights_size(cfg) elements) to the device,
+ * allocates every cache and workspace, and marks every view cold.
+ * On failure *out is NULL and the code says why. */
+int ivit_create(const ivit_config* cfg, const uint16_t* weights_bf16_host,
+                ivit_handle** out);
+
+/* Full encode of one frame per view (the paper's full forward that seeds the
+ * reference, Sec. III-B).  frames_dev: uint8 [SV][img_h][img_w][3].
+ * tokens_out_dev: bf16 [SV][N][D] final tokens (after the final LN), or NULL.
+ * Re-seeds every cache and reference and marks every view warm. */
+int ivit_encode_full(ivit_handle* h, const uint8_t* frames_dev, uint16_t* tokens_out_dev,
+                     void* stream);
+
+/* Incremental encode (Sec. III-B, Eq. 3-5): scores every token's patch embedding
+ * against its reference (cosine, fp32), selects the tokens to update per view, runs
+ * every block on those tokens only (their queries attend over all N tokens of the
+ * view, the others' K/V come from the cache), and returns all tokens: updated ones
+ * recomputed, the rest from the final-token cache.  A cold view updates every token.
+ * tokens_out_dev: bf16 [SV][N][D] or NULL.  changed_count_dev: int32 [SV] number of
+ * updated tokens per view, or NULL.  No host synchronisation happens inside. */
+int ivit_encode_incremental(ivit_handle* h, const uint8_t* frames_dev,
+                            uint16_t* tokens_out_dev, int32_t* changed_count_dev,
+                            void* stream);
+
+/* Copies the ascending updated-token list of view `sv` from the last encode call:
+ * idx_dev int32 [N] (first *count entries valid), count_dev int32 [1] (either may be
+ * NULL).  Enqueued on `stream`. */
+int ivit_get_changed(ivit_handle* h, int sv, int32_t* idx_dev, int32_t* count_dev,
+                     void* stream);
+
+/* Copies per-view state for inspection: which = 0 key cache of `layer`, 1 value cache
+ * of `layer`, 2 final-token cache (all bf16 [SV][N][D]), 3 reference embeddings
+ * (fp32 [SV][N][D]).  dst_dev must hold that many bytes. */
+int ivit_get_cache(ivit_handle* h, int which, int layer, void* dst_dev, void* stream);
+
+/* Marks the views of camera stream `stream_index` (all streams if -1) cold: the next
+ * incremental call recomputes every token of those views.  Host-side only. */
+int ivit_reset(ivit_handle* h, int stream_index);
+
+/* Kernel timing hook: when enabled, every launch of the dominant kernel family (the
+ * tensor-core GEMM) is bracketed by CUDA events on the launch stream; the sum and
+ * count since the last call are returned and reset. */
+int ivit_profile_enable(ivit_handle* h, int enable);
+int ivit_profile_read(ivit_handle* h, double* gemm_ms_total, int64_t* gemm_launches,
+                      double* gemm_bytes_total);
+
+/* Reads and clears the device error word (0 = none; nonzero = a kernel's bounded
+ * wait expired, the kernel skipped its work and returned).  Synchronises `stream`. */
+int ivit_device_status(ivit_handle* h, void* stream);
+
+/* Number of the library's kernel launches made by the last encode call. */
+int64_t ivit_last_launch_count(const ivit_handle* h);
+
+void ivit_destroy(ivit_handle* h);
+
+/* Message of the last failure on `h` (or of the last failed create if h is NULL). */
+const char* ivit_last_error(const ivit_handle* h);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* IVIT_H */

@@ -1,0 +1,629 @@
+// Engine behind the C ABI of include/ivit.h: weight upload, per-view caches,
+// workspaces, TMA descriptors and the per-frame launch chain of temporal token reuse
+// (Sec. III-B): embed -> score (Eq. 3) -> select/compact -> gather -> per layer
+// {LN1, QKV + K/V cache scatter (Eq. 4-5), attention of updated queries over all
+// tokens, out-proj + residual, LN2, MLP up + GELU, MLP down + residual} -> final LN
+// scattered into the final-token cache -> output copy.
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/ivit.h"
+#include "internal.h"
+#include "ptx.cuh"
+
+using ivit::bf16;
+
+namespace {
+
+struct LayerW {
+  bf16 *wqkv, *wo, *w1, *w2;
+  float *bqkv, *bo, *b1, *b2, *ln1g, *ln1b, *ln2g, *ln2b;
+  CUtensorMap tm_qkv, tm_o, tm_1, tm_2;
+};
+
+struct EventPair {
+  cudaEvent_t a, b;
+};
+
+thread_local std::string g_create_error;
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// bf16 2-D tensor [rows][inner] with the given row stride; box = box_inner x box_rows,
+// 128-byte swizzle (box_inner * 2 == 128), out-of-bounds elements read as zero.
+bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t stride_bytes,
+              uint32_t box_inner, uint32_t box_rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {inner, rows};
+  cuuint64_t strides[1] = {stride_bytes};
+  cuuint32_t box[2] = {box_inner, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Bump allocator over one device allocation; every sub-buffer 256-byte aligned.
+struct Arena {
+  size_t size = 0;
+  char* base = nullptr;
+  size_t take(size_t bytes) {
+    const size_t off = size;
+    size += (bytes + 255) & ~static_cast<size_t>(255);
+    return off;
+  }
+  template <class T>
+  T* at(size_t off) const {
+    return reinterpret_cast<T*>(base + off);
+  }
+};
+
+inline float bf16_bits_to_float(uint16_t b) {
+  uint32_t u = static_cast<uint32_t>(b) << 16;
+  float f;
+  std::memcpy(&f, &u, 4);
+  return f;
+}
+
+}  // namespace
+
+struct ivit_handle {
+  ivit_config cfg{};
+  int N = 0, D = 0, F = 0, H = 0, L = 0, SV = 0, Kp = 0, KPAD = 0, M_max = 0;
+  int device = 0, num_sms = 0;
+  int grid64 = 0, grid256 = 0, row_grid = 0, bn_embed = 256, bn_inc = 64;
+  size_t ws_bytes = 0;
+
+  void* wmem = nullptr;  // weights (device)
+  void* smem = nullptr;  // state + workspaces (device)
+  bf16* w_pe = nullptr;
+  float *b_pe = nullptr, *pos = nullptr, *lnfg = nullptr, *lnfb = nullptr;
+  std::vector<LayerW> layers;
+  CUtensorMap tm_pe, tm_patches, tm_xn, tm_o, tm_h;
+
+  bf16* patches = nullptr;
+  float *e_t = nullptr, *e_ref = nullptr, *sims = nullptr, *x = nullptr, *ws = nullptr;
+  int *idx = nullptr, *counts = nullptr, *cu_rows = nullptr, *rowtok = nullptr, *done_ctr = nullptr;
+  int *tile_ctr = nullptr, *err = nullptr;
+  bf16 *xn = nullptr, *q = nullptr, *o = nullptr, *hbuf = nullptr, *cacheK = nullptr,
+       *cacheV = nullptr, *tok_out = nullptr;
+
+  std::vector<uint8_t> cold;
+  int64_t launches = 0;
+
+  bool profiling = false;
+  std::vector<EventPair> prof_events;
+  size_t prof_used = 0;
+  double prof_bytes = 0.0;
+  std::vector<double> call_static_bytes;  // per GEMM of the current call: weight bytes etc.
+
+  std::string error;
+
+  int fail(int code, const std::string& msg) {
+    error = msg;
+    return code;
+  }
+  int cuda_fail(const char* what, cudaError_t e) {
+    error = std::string(what) + ": " + cudaGetErrorString(e);
+    return e == cudaErrorMemoryAllocation ? IVIT_ERR_OOM : IVIT_ERR_CUDA;
+  }
+};
+
+#define IVIT_CK(h, call)                                 \
+  do {                                                   \
+    cudaError_t e_ = (call);                             \
+    if (e_ != cudaSuccess) return (h)->cuda_fail(#call, e_); \
+  } while (0)
+
+namespace {
+
+const char* validate(const ivit_config* c) {
+  if (!c) return "null config";
+  if (c->patch <= 0 || c->img_h <= 0 || c->img_w <= 0) return "patch and image size must be positive";
+  if (c->img_h % c->patch || c->img_w % c->patch) return "patch must divide img_h and img_w";
+  const long long n = static_cast<long long>(c->img_h / c->patch) * (c->img_w / c->patch);
+  if (n > 1024) return "at most 1024 tokens per view";
+  if (c->dim <= 0 || c->dim % 64) return "dim must be a positive multiple of 64";
+  if (c->heads <= 0 || c->dim % c->heads) return "heads must divide dim";
+  const int dh = c->dim / c->heads;
+  if (dh % 8 || dh > 128) return "head_dim must be a multiple of 8 and at most 128";
+  if (c->depth <= 0) return "depth must be positive";
+  if (c->mlp_dim <= 0 || c->mlp_dim % 8) return "mlp_dim must be a positive multiple of 8";
+  if (c->n_streams <= 0 || c->n_views <= 0) return "n_streams and n_views must be positive";
+  if (static_cast<long long>(c->n_streams) * c->n_views > 4096) return "at most 4096 views";
+  if (!(c->ln_eps > 0.f)) return "ln_eps must be positive";
+  if (c->gelu != IVIT_GELU_TANH && c->gelu != IVIT_GELU_ERF) return "bad gelu";
+  if (c->select_mode != IVIT_SEL_THRESHOLD && c->select_mode != IVIT_SEL_TOPK) return "bad select_mode";
+  if (c->ref_mode != IVIT_REF_PREV_FRAME && c->ref_mode != IVIT_REF_LAST_REFRESH) return "bad ref_mode";
+  if (c->select_mode == IVIT_SEL_TOPK && c->topk < 0) return "topk must be >= 0";
+  if (!std::isfinite(c->threshold)) return "threshold must be finite";
+  return nullptr;
+}
+
+size_t weights_count(const ivit_config* c) {
+  const size_t D = c->dim, F = c->mlp_dim, N = static_cast<size_t>(c->img_h / c->patch) * (c->img_w / c->patch);
+  const size_t Kp = static_cast<size_t>(c->patch) * c->patch * 3;
+  const size_t per_layer = 2 * D + 3 * D * D + 3 * D + D * D + D + 2 * D + F * D + F + D * F + D;
+  return D * Kp + D + N * D + per_layer * c->depth + 2 * D;
+}
+
+int setup(ivit_handle* h, const uint16_t* wb) {
+  const ivit_config& c = h->cfg;
+  h->N = (c.img_h / c.patch) * (c.img_w / c.patch);
+  h->D = c.dim;
+  h->F = c.mlp_dim;
+  h->H = c.heads;
+  h->L = c.depth;
+  h->SV = c.n_streams * c.n_views;
+  h->Kp = c.patch * c.patch * 3;
+  h->KPAD = (h->Kp + 63) / 64 * 64;
+  h->M_max = h->SV * h->N;
+  h->cold.assign(h->SV, 1);
+  const size_t D = h->D, F = h->F, N = h->N, L = h->L, M = h->M_max;
+
+  IVIT_CK(h, cudaGetDevice(&h->device));
+  IVIT_CK(h, cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device));
+  IVIT_CK(h, ivit::gemm_setup(64));
+  IVIT_CK(h, ivit::gemm_setup(256));
+  h->grid64 = h->num_sms * ivit::gemm_ctas_per_sm(64);
+  h->grid256 = h->num_sms * ivit::gemm_ctas_per_sm(256);
+  h->row_grid = h->num_sms * 4;
+  h->bn_embed = M <= 64 ? 64 : 256;
+  h->bn_inc = M <= 1024 ? 64 : 256;
+  h->ws_bytes = std::max(static_cast<size_t>(h->grid64) * 64, static_cast<size_t>(h->grid256) * 256) *
+                128 * sizeof(float);
+
+  // ---- weights: bf16 matrices (W_pe padded to KPAD columns), fp32 vectors
+  Arena wa;
+  const size_t o_pe = wa.take(D * h->KPAD * 2), o_bpe = wa.take(D * 4), o_pos = wa.take(N * D * 4);
+  struct LOff { size_t qkv, o, w1, w2, bqkv, bo, b1, b2, g1, be1, g2, be2; };
+  std::vector<LOff> lo(L);
+  for (size_t l = 0; l < L; ++l) {
+    lo[l].qkv = wa.take(3 * D * D * 2);
+    lo[l].o = wa.take(D * D * 2);
+    lo[l].w1 = wa.take(F * D * 2);
+    lo[l].w2 = wa.take(D * F * 2);
+    lo[l].bqkv = wa.take(3 * D * 4);
+    lo[l].bo = wa.take(D * 4);
+    lo[l].b1 = wa.take(F * 4);
+    lo[l].b2 = wa.take(D * 4);
+    lo[l].g1 = wa.take(D * 4);
+    lo[l].be1 = wa.take(D * 4);
+    lo[l].g2 = wa.take(D * 4);
+    lo[l].be2 = wa.take(D * 4);
+  }
+  const size_t o_gf = wa.take(D * 4), o_bf = wa.take(D * 4);
+
+  std::vector<char> host(wa.size, 0);
+  auto put_bf16 = [&](size_t off, const uint16_t* src, size_t rows, size_t cols, size_t ld) {
+    for (size_t r = 0; r < rows; ++r) std::memcpy(&host[off + r * ld * 2], src + r * cols, cols * 2);
+  };
+  auto put_f32 = [&](size_t off, const uint16_t* src, size_t n) {
+    float* dst = reinterpret_cast<float*>(&host[off]);
+    for (size_t i = 0; i < n; ++i) dst[i] = bf16_bits_to_float(src[i]);
+  };
+  const uint16_t* p = wb;
+  put_bf16(o_pe, p, D, h->Kp, h->KPAD); p += D * h->Kp;
+  put_f32(o_bpe, p, D); p += D;
+  put_f32(o_pos, p, N * D); p += N * D;
+  for (size_t l = 0; l < L; ++l) {
+    put_f32(lo[l].g1, p, D); p += D;
+    put_f32(lo[l].be1, p, D); p += D;
+    put_bf16(lo[l].qkv, p, 3 * D, D, D); p += 3 * D * D;
+    put_f32(lo[l].bqkv, p, 3 * D); p += 3 * D;
+    put_bf16(lo[l].o, p, D, D, D); p += D * D;
+    put_f32(lo[l].bo, p, D); p += D;
+    put_f32(lo[l].g2, p, D); p += D;
+    put_f32(lo[l].be2, p, D); p += D;
+    put_bf16(lo[l].w1, p, F, D, D); p += F * D;
+    put_f32(lo[l].b1, p, F); p += F;
+    put_bf16(lo[l].w2, p, D, F, F); p += D * F;
+    put_f32(lo[l].b2, p, D); p += D;
+  }
+  put_f32(o_gf, p, D); p += D;
+  put_f32(o_bf, p, D); p += D;
+
+  IVIT_CK(h, cudaMalloc(&h->wmem, wa.size));
+  IVIT_CK(h, cudaMemcpy(h->wmem, host.data(), wa.size, cudaMemcpyHostToDevice));
+  wa.base = static_cast<char*>(h->wmem);
+  h->w_pe = wa.at<bf16>(o_pe);
+  h->b_pe = wa.at<float>(o_bpe);
+  h->pos = wa.at<float>(o_pos);
+  h->lnfg = wa.at<float>(o_gf);
+  h->lnfb = wa.at<float>(o_bf);
+  h->layers.resize(L);
+  for (size_t l = 0; l < L; ++l) {
+    LayerW& w = h->layers[l];
+    w.wqkv = wa.at<bf16>(lo[l].qkv);
+    w.wo = wa.at<bf16>(lo[l].o);
+    w.w1 = wa.at<bf16>(lo[l].w1);
+    w.w2 = wa.at<bf16>(lo[l].w2);
+    w.bqkv = wa.at<float>(lo[l].bqkv);
+    w.bo = wa.at<float>(lo[l].bo);
+    w.b1 = wa.at<float>(lo[l].b1);
+    w.b2 = wa.at<float>(lo[l].b2);
+    w.ln1g = wa.at<float>(lo[l].g1);
+    w.ln1b = wa.at<float>(lo[l].be1);
+    w.ln2g = wa.at<float>(lo[l].g2);
+    w.ln2b = wa.at<float>(lo[l].be2);
+    if (!make_map(&w.tm_qkv, w.wqkv, D, 3 * D, D * 2, 64, 128) ||
+        !make_map(&w.tm_o, w.wo, D, D, D * 2, 64, 128) ||
+        !make_map(&w.tm_1, w.w1, D, F, D * 2, 64, 128) ||
+        !make_map(&w.tm_2, w.w2, F, D, F * 2, 64, 128))
+      return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for a weight matrix");
+  }
+  if (!make_map(&h->tm_pe, h->w_pe, h->KPAD, D, h->KPAD * 2, 64, 128))
+    return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for W_pe");
+
+  // ---- state and workspaces
+  Arena sa;
+  const size_t o_patch = sa.take(M * h->KPAD * 2), o_et = sa.take(M * D * 4), o_er = sa.take(M * D * 4);
+  const size_t o_sims = sa.take(M * 4), o_idx = sa.take(M * 4), o_cnt = sa.take(h->SV * 4);
+  const size_t o_cu = sa.take((h->SV + 1) * 4), o_rt = sa.take(M * 4), o_done = sa.take(4);
+  const size_t o_x = sa.take(M * D * 4), o_xn = sa.take(M * D * 2), o_q = sa.take(M * D * 2);
+  const size_t o_o = sa.take(M * D * 2), o_h = sa.take(M * F * 2);
+  const size_t o_ck = sa.take(L * M * D * 2), o_cv = sa.take(L * M * D * 2), o_tok = sa.take(M * D * 2);
+  const size_t o_ws = sa.take(h->ws_bytes), o_tc = sa.take((h->grid64 + h->grid256) * 4);
+  const size_t o_err = sa.take(4);
+  IVIT_CK(h, cudaMalloc(&h->smem, sa.size));
+  IVIT_CK(h, cudaMemset(h->smem, 0, sa.size));
+  sa.base = static_cast<char*>(h->smem);
+  h->patches = sa.at<bf16>(o_patch);
+  h->e_t = sa.at<float>(o_et);
+  h->e_ref = sa.at<float>(o_er);
+  h->sims = sa.at<float>(o_sims);
+  h->idx = sa.at<int>(o_idx);
+  h->counts = sa.at<int>(o_cnt);
+  h->cu_rows = sa.at<int>(o_cu);
+  h->rowtok = sa.at<int>(o_rt);
+  h->done_ctr = sa.at<int>(o_done);
+  h->x = sa.at<float>(o_x);
+  h->xn = sa.at<bf16>(o_xn);
+  h->q = sa.at<bf16>(o_q);
+  h->o = sa.at<bf16>(o_o);
+  h->hbuf = sa.at<bf16>(o_h);
+  h->cacheK = sa.at<bf16>(o_ck);
+  h->cacheV = sa.at<bf16>(o_cv);
+  h->tok_out = sa.at<bf16>(o_tok);
+  h->ws = sa.at<float>(o_ws);
+  h->tile_ctr = sa.at<int>(o_tc);
+  h->err = sa.at<int>(o_err);
+  if (!make_map(&h->tm_patches, h->patches, h->KPAD, M, h->KPAD * 2, 64, 32) ||
+      !make_map(&h->tm_xn, h->xn, D, M, D * 2, 64, 32) ||
+      !make_map(&h->tm_o, h->o, D, M, D * 2, 64, 32) ||
+      !make_map(&h->tm_h, h->hbuf, F, M, F * 2, 64, 32))
+    return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
+  IVIT_CK(h, cudaDeviceSynchronize());
+  return IVIT_OK;
+}
+
+void release(ivit_handle* h) {
+  if (h->wmem) cudaFree(h->wmem);
+  if (h->smem) cudaFree(h->smem);
+  for (auto& e : h->prof_events) {
+    cudaEventDestroy(e.a);
+    cudaEventDestroy(e.b);
+  }
+  h->wmem = h->smem = nullptr;
+  h->prof_events.clear();
+}
+
+// Algorithmic bytes of one GEMM launch at M rows (weights, input rows, output rows, bias).
+double gemm_bytes(int n_out, int k, int kind, long long M) {
+  const double out_b = kind == ivit::kEpiF32Bias ? 4.0 : kind == ivit::kEpiResid ? 8.0 : 2.0;
+  return 2.0 * n_out * k + 2.0 * M * k + out_b * M * n_out + 4.0 * n_out;
+}
+
+int gemm(ivit_handle* h, int bn, const CUtensorMap& tw, const CUtensorMap& tx, ivit::GemmArgs a,
+         cudaStream_t s) {
+  a.err = h->err;
+  a.tile_ctr = h->tile_ctr;
+  a.ws = h->ws;
+  a.ws_items = static_cast<int>(h->ws_bytes / (static_cast<size_t>(bn) * 128 * sizeof(float)));
+  a.max_splits = 16;
+  const int grid = bn == 64 ? h->grid64 : h->grid256;
+  EventPair* ev = nullptr;
+  if (h->profiling) {
+    if (h->prof_used == h->prof_events.size()) {
+      EventPair e{};
+      IVIT_CK(h, cudaEventCreate(&e.a));
+      IVIT_CK(h, cudaEventCreate(&e.b));
+      h->prof_events.push_back(e);
+    }
+    ev = &h->prof_events[h->prof_used++];
+    IVIT_CK(h, cudaEventRecord(ev->a, s));
+  }
+  IVIT_CK(h, ivit::launch_gemm(bn, tw, tx, a, grid, false, s));
+  ++h->launches;
+  if (ev) {
+    IVIT_CK(h, cudaEventRecord(ev->b, s));
+    h->call_static_bytes.push_back(a.n_out);  // n_out, k, kind, static M (or -1)
+    h->call_static_bytes.push_back(a.k);
+    h->call_static_bytes.push_back(a.epi.kind);
+    h->call_static_bytes.push_back(a.d_rows ? -1.0 : static_cast<double>(a.m_static));
+  }
+  return IVIT_OK;
+}
+
+int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_counts, bool full,
+        cudaStream_t s) {
+  const ivit_config& c = h->cfg;
+  const int N = h->N, D = h->D, F = h->F, SV = h->SV, M = h->M_max;
+  ivit::ColdMask cm;
+  std::memset(&cm, 0, sizeof cm);
+  for (int v = 0; v < SV; ++v)
+    if (full || h->cold[v]) cm.bits[v >> 5] |= 1u << (v & 31);
+  const int bn = full ? 256 : h->bn_inc;
+  const int* total = h->cu_rows + SV;
+  h->launches = 0;
+  h->call_static_bytes.clear();
+
+  IVIT_CK(h, ivit::launch_patchify(frames, h->patches, SV, c.img_h, c.img_w, c.patch, h->KPAD, s));
+  ++h->launches;
+  {
+    ivit::GemmArgs a;
+    a.n_out = D;
+    a.k = h->KPAD;
+    a.m_static = M;
+    a.epi.kind = ivit::kEpiF32Bias;
+    a.epi.bias = h->b_pe;
+    a.epi.out_f32 = h->e_t;
+    a.epi.ld_out = D;
+    if (int r = gemm(h, h->bn_embed, h->tm_pe, h->tm_patches, a, s)) return r;
+  }
+  if (!full) {
+    IVIT_CK(h, ivit::launch_score(h->e_t, h->e_ref, h->sims, M, D, c.ref_mode == IVIT_REF_PREV_FRAME, s));
+    ++h->launches;
+  }
+  IVIT_CK(h, ivit::launch_select(h->sims, N, SV, full ? IVIT_SEL_THRESHOLD : c.select_mode, c.threshold,
+                                 c.topk, cm, h->idx, h->counts, h->cu_rows, h->rowtok, h->done_ctr,
+                                 user_counts, s));
+  ++h->launches;
+  IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, h->x, h->e_ref, N, D,
+                                 c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
+  ++h->launches;
+
+  for (int l = 0; l < h->L; ++l) {
+    const LayerW& w = h->layers[l];
+    bf16* ck = h->cacheK + static_cast<size_t>(l) * M * D;
+    bf16* cv = h->cacheV + static_cast<size_t>(l) * M * D;
+    IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln1g, w.ln1b, h->xn, nullptr, D, c.ln_eps, M,
+                                      h->row_grid, s));
+    ++h->launches;
+    {
+      ivit::GemmArgs a;
+      a.n_out = 3 * D;
+      a.k = D;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiQKV;
+      a.epi.bias = w.bqkv;
+      a.epi.out_bf16 = h->q;
+      a.epi.ld_out = D;
+      a.epi.cache_k = ck;
+      a.epi.cache_v = cv;
+      a.epi.rowtok = h->rowtok;
+      a.epi.dim = D;
+      if (int r = gemm(h, bn, w.tm_qkv, h->tm_xn, a, s)) return r;
+    }
+    IVIT_CK(h, ivit::launch_attention(h->q, ck, cv, h->cu_rows, h->o, SV, N, D, h->H, s));
+    ++h->launches;
+    {
+      ivit::GemmArgs a;
+      a.n_out = D;
+      a.k = D;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiResid;
+      a.epi.bias = w.bo;
+      a.epi.out_f32 = h->x;
+      a.epi.ld_out = D;
+      if (int r = gemm(h, bn, w.tm_o, h->tm_o, a, s)) return r;
+    }
+    IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln2g, w.ln2b, h->xn, nullptr, D, c.ln_eps, M,
+                                      h->row_grid, s));
+    ++h->launches;
+    {
+      ivit::GemmArgs a;
+      a.n_out = F;
+      a.k = D;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiGelu;
+      a.epi.bias = w.b1;
+      a.epi.out_bf16 = h->hbuf;
+      a.epi.ld_out = F;
+      a.epi.gelu_mode = c.gelu;
+      if (int r = gemm(h, bn, w.tm_1, h->tm_xn, a, s)) return r;
+    }
+    {
+      ivit::GemmArgs a;
+      a.n_out = D;
+      a.k = F;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiResid;
+      a.epi.bias = w.b2;
+      a.epi.out_f32 = h->x;
+      a.epi.ld_out = D;
+      if (int r = gemm(h, bn, w.tm_2, h->tm_h, a, s)) return r;
+    }
+  }
+  IVIT_CK(h, ivit::launch_layernorm(total, h->x, h->lnfg, h->lnfb, h->tok_out, h->rowtok, D, c.ln_eps,
+                                    M, h->row_grid, s));
+  ++h->launches;
+  if (out)
+    IVIT_CK(h, cudaMemcpyAsync(out, h->tok_out, static_cast<size_t>(M) * D * 2, cudaMemcpyDeviceToDevice, s));
+  for (int v = 0; v < SV; ++v) h->cold[v] = 0;
+
+  if (h->profiling) {
+    int rows = 0;
+    IVIT_CK(h, cudaMemcpyAsync(&rows, total, sizeof(int), cudaMemcpyDeviceToHost, s));
+    IVIT_CK(h, cudaStreamSynchronize(s));
+    for (size_t i = 0; i + 3 < h->call_static_bytes.size(); i += 4) {
+      const double m = h->call_static_bytes[i + 3] >= 0 ? h->call_static_bytes[i + 3] : rows;
+      h->prof_bytes += gemm_bytes(static_cast<int>(h->call_static_bytes[i]),
+                                  static_cast<int>(h->call_static_bytes[i + 1]),
+                                  static_cast<int>(h->call_static_bytes[i + 2]), static_cast<long long>(m));
+    }
+  }
+  return IVIT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t ivit_weights_size(const ivit_config* cfg) {
+  if (validate(cfg)) return 0;
+  return weights_count(cfg);
+}
+
+int ivit_create(const ivit_config* cfg, const uint16_t* weights_bf16_host, ivit_handle** out) {
+  if (!out) {
+    g_create_error = "null output pointer";
+    return IVIT_ERR_ARG;
+  }
+  *out = nullptr;
+  if (const char* why = validate(cfg)) {
+    g_create_error = why;
+    return cfg ? IVIT_ERR_SHAPE : IVIT_ERR_ARG;
+  }
+  if (!weights_bf16_host) {
+    g_create_error = "null weights";
+    return IVIT_ERR_ARG;
+  }
+  ivit_handle* h = new (std::nothrow) ivit_handle();
+  if (!h) {
+    g_create_error = "host allocation failed";
+    return IVIT_ERR_OOM;
+  }
+  h->cfg = *cfg;
+  const int r = setup(h, weights_bf16_host);
+  if (r != IVIT_OK) {
+    g_create_error = h->error;
+    release(h);
+    delete h;
+    return r;
+  }
+  *out = h;
+  return IVIT_OK;
+}
+
+int ivit_encode_full(ivit_handle* h, const uint8_t* frames_dev, uint16_t* tokens_out_dev, void* stream) {
+  if (!h) return IVIT_ERR_ARG;
+  if (!frames_dev) return h->fail(IVIT_ERR_ARG, "null frames");
+  return run(h, frames_dev, tokens_out_dev, nullptr, true, static_cast<cudaStream_t>(stream));
+}
+
+int ivit_encode_incremental(ivit_handle* h, const uint8_t* frames_dev, uint16_t* tokens_out_dev,
+                            int32_t* changed_count_dev, void* stream) {
+  if (!h) return IVIT_ERR_ARG;
+  if (!frames_dev) return h->fail(IVIT_ERR_ARG, "null frames");
+  return run(h, frames_dev, tokens_out_dev, changed_count_dev, false, static_cast<cudaStream_t>(stream));
+}
+
+int ivit_get_changed(ivit_handle* h, int sv, int32_t* idx_dev, int32_t* count_dev, void* stream) {
+  if (!h) return IVIT_ERR_ARG;
+  if (sv < 0 || sv >= h->SV) return h->fail(IVIT_ERR_ARG, "view index out of range");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (idx_dev)
+    IVIT_CK(h, cudaMemcpyAsync(idx_dev, h->idx + static_cast<size_t>(sv) * h->N, h->N * sizeof(int),
+                               cudaMemcpyDeviceToDevice, s));
+  if (count_dev)
+    IVIT_CK(h, cudaMemcpyAsync(count_dev, h->counts + sv, sizeof(int), cudaMemcpyDeviceToDevice, s));
+  return IVIT_OK;
+}
+
+int ivit_get_cache(ivit_handle* h, int which, int layer, void* dst_dev, void* stream) {
+  if (!h) return IVIT_ERR_ARG;
+  if (!dst_dev) return h->fail(IVIT_ERR_ARG, "null destination");
+  const size_t elems = static_cast<size_t>(h->M_max) * h->D;
+  const void* src = nullptr;
+  size_t bytes = elems * 2;
+  if (which == 0 || which == 1) {
+    if (layer < 0 || layer >= h->L) return h->fail(IVIT_ERR_ARG, "layer out of range");
+    src = (which == 0 ? h->cacheK : h->cacheV) + static_cast<size_t>(layer) * elems;
+  } else if (which == 2) {
+    src = h->tok_out;
+  } else if (which == 3) {
+    src = h->e_ref;
+    bytes = elems * 4;
+  } else {
+    return h->fail(IVIT_ERR_ARG, "bad cache selector");
+  }
+  IVIT_CK(h, cudaMemcpyAsync(dst_dev, src, bytes, cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream)));
+  return IVIT_OK;
+}
+
+int ivit_reset(ivit_handle* h, int stream_index) {
+  if (!h) return IVIT_ERR_ARG;
+  if (stream_index < -1 || stream_index >= h->cfg.n_streams)
+    return h->fail(IVIT_ERR_ARG, "stream index out of range");
+  for (int v = 0; v < h->SV; ++v)
+    if (stream_index == -1 || v / h->cfg.n_views == stream_index) h->cold[v] = 1;
+  return IVIT_OK;
+}
+
+int ivit_profile_enable(ivit_handle* h, int enable) {
+  if (!h) return IVIT_ERR_ARG;
+  h->profiling = enable != 0;
+  h->prof_used = 0;
+  h->prof_bytes = 0.0;
+  return IVIT_OK;
+}
+
+int ivit_profile_read(ivit_handle* h, double* gemm_ms_total, int64_t* gemm_launches,
+                      double* gemm_bytes_total) {
+  if (!h) return IVIT_ERR_ARG;
+  double ms = 0.0;
+  for (size_t i = 0; i < h->prof_used; ++i) {
+    IVIT_CK(h, cudaEventSynchronize(h->prof_events[i].b));
+    float t = 0.f;
+    IVIT_CK(h, cudaEventElapsedTime(&t, h->prof_events[i].a, h->prof_events[i].b));
+    ms += t;
+  }
+  if (gemm_ms_total) *gemm_ms_total = ms;
+  if (gemm_launches) *gemm_launches = static_cast<int64_t>(h->prof_used);
+  if (gemm_bytes_total) *gemm_bytes_total = h->prof_bytes;
+  h->prof_used = 0;
+  h->prof_bytes = 0.0;
+  return IVIT_OK;
+}
+
+int ivit_device_status(ivit_handle* h, void* stream) {
+  if (!h) return IVIT_ERR_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int word = 0;
+  IVIT_CK(h, cudaMemcpyAsync(&word, h->err, sizeof(int), cudaMemcpyDeviceToHost, s));
+  IVIT_CK(h, cudaMemsetAsync(h->err, 0, sizeof(int), s));
+  IVIT_CK(h, cudaStreamSynchronize(s));
+  return word;
+}
+
+int64_t ivit_last_launch_count(const ivit_handle* h) { return h ? h->launches : 0; }
+
+void ivit_destroy(ivit_handle* h) {
+  if (!h) return;
+  release(h);
+  delete h;
+}
+
+const char* ivit_last_error(const ivit_handle* h) {
+  return h ? h->error.c_str() : g_create_error.c_str();
+}
+
+}  // extern "C"

@@ -1,0 +1,92 @@
+// Kernel launch interfaces shared by the engine and the kernel translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ivit {
+
+using bf16 = __nv_bfloat16;
+
+// ------------------------------------------------------------------ GEMM (tcgen05)
+// Y[r][f] = sum_k X[r][k] * W[f][k] for r < M rows, f < Nout features, then an
+// epilogue.  W is the weight matrix in Linear layout [Nout][K] (bf16, K-major), X the
+// packed activation rows [M][K] (bf16, K-major).
+enum EpiKind : int {
+  kEpiF32Bias = 0,  // out_f32[r][f] = y + bias[f]
+  kEpiQKV = 1,      // f <  D: out_bf16[r][f] = y + b (queries, packed rows)
+                    // f < 2D: cache_k[rowtok[r]][f-D], else cache_v[rowtok[r]][f-2D]  (Eq. 5)
+  kEpiResid = 2,    // out_f32[r][f] += y + bias[f]  (residual stream, fp32)
+  kEpiGelu = 3,     // out_bf16[r][f] = gelu(y + bias[f])
+};
+
+struct GemmEpilogue {
+  int kind = kEpiF32Bias;
+  const float* bias = nullptr;   // [Nout]
+  float* out_f32 = nullptr;      // kEpiF32Bias / kEpiResid, row stride ld_out
+  bf16* out_bf16 = nullptr;      // kEpiGelu / kEpiQKV (queries), row stride ld_out
+  bf16* cache_k = nullptr;       // kEpiQKV: this layer's key cache [SV*N][D]
+  bf16* cache_v = nullptr;       // kEpiQKV: this layer's value cache [SV*N][D]
+  const int* rowtok = nullptr;   // kEpiQKV: packed row -> token index v*N + i
+  int dim = 0;                   // kEpiQKV: D
+  int gelu_mode = 0;             // kEpiGelu: 0 tanh form, 1 erf form
+  int ld_out = 0;
+};
+
+struct GemmArgs {
+  int n_out = 0;                 // Nout
+  int k = 0;                     // K
+  const int* d_rows = nullptr;   // device row count M (nullptr: use m_static)
+  int m_static = 0;
+  int max_splits = 16;
+  float* ws = nullptr;           // split-K partials, ws_items x (bn_max x 128) fp32
+  int ws_items = 0;
+  int* tile_ctr = nullptr;       // one arrival counter per output tile, zero between launches
+  int* err = nullptr;            // device error word
+  GemmEpilogue epi;
+};
+
+// Returns the dynamic shared memory size (bytes) of the GEMM variant.
+size_t gemm_smem_bytes(int bn_max);
+// One-time attribute setup (dynamic smem opt-in).  Returns a CUDA error.
+cudaError_t gemm_setup(int bn_max);
+// Occupancy of the variant (CTAs per SM).
+int gemm_ctas_per_sm(int bn_max);
+cudaError_t launch_gemm(int bn_max, const CUtensorMap& tm_w, const CUtensorMap& tm_x,
+                        const GemmArgs& a, int grid, bool pdl, cudaStream_t s);
+
+// ------------------------------------------------------------------- other kernels
+struct ColdMask {
+  uint32_t bits[128];  // bit v set: view v is cold (updates every token); up to 4096 views
+};
+
+cudaError_t launch_patchify(const uint8_t* frames, bf16* patches, int sv, int img_h, int img_w,
+                            int patch, int kpad, cudaStream_t s);
+
+cudaError_t launch_score(const float* e_t, float* e_ref, float* sims, int rows, int dim,
+                         int copy_ref, cudaStream_t s);
+
+cudaError_t launch_select(const float* sims, int n_tok, int sv, int mode, float tau, int topk,
+                          const ColdMask& cold, int* idx, int* counts, int* cu_rows, int* rowtok,
+                          int* done_ctr, int* user_counts, cudaStream_t s);
+
+cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const float* e_t,
+                          const float* pos, float* x, float* e_ref, int n_tok, int dim,
+                          int ref_last_refresh, const ColdMask& cold, int max_rows, int grid,
+                          cudaStream_t s);
+
+// y[r] = LN(x[r]) (bf16) for r < *rows; when dst_rowtok is set, row r is written to
+// row dst_rowtok[r] of y instead (final-token cache scatter).
+cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma, const float* beta,
+                             bf16* y, const int* dst_rowtok, int dim, float eps, int max_rows,
+                             int grid, cudaStream_t s);
+
+// O[r] = softmax(Q[r] K_v^T / sqrt(dh)) V_v per head, for the packed query rows r of
+// each view v (cu_rows), over the N cached keys/values of that view.
+cudaError_t launch_attention(const bf16* q, const bf16* cache_k, const bf16* cache_v,
+                             const int* cu_rows, bf16* o, int sv, int n_tok, int dim, int heads,
+                             cudaStream_t s);
+
+}  // namespace ivit

@@ -1,0 +1,75 @@
+"""The C-ABI library loads without a GPU, exports every entry point that
+include/ivit.h declares, and rejects bad configurations before touching the device."""
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+from paper_2607_12287_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def pkg():
+    from paper_2607_12287_gb300 import build
+    build.build()
+    import paper_2607_12287_gb300 as p
+    p.load()
+    return p
+
+
+def declared_entry_points():
+    text = open(os.path.join(ROOT, "include", "ivit.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(ivit_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_binding_names(pkg):
+    assert declared_entry_points() == sorted(pkg.EXPORTED)
+
+
+def test_library_exports_every_declared_symbol(pkg):
+    out = subprocess.run(["nm", "-D", "--defined-only", pkg.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (ivit_[a-z_]+)$", out, flags=re.M))
+    missing = set(declared_entry_points()) - exported
+    assert not missing, f"missing symbols: {missing}"
+
+
+def test_weights_size_matches_generator_layout(pkg):
+    for shape in (synth.VIT_TINY_224, synth.SO400M_224, synth.SO400M_448):
+        assert pkg.ivit_weights_size(pkg.make_config(shape)) == synth.weight_count(shape)
+
+
+@pytest.mark.parametrize("field,value", [
+    ("dim", 100), ("heads", 7), ("patch", 15), ("mlp_dim", 1001), ("depth", 0),
+    ("n_views", 0), ("gelu", 5), ("select_mode", 9), ("ref_mode", 3), ("ln_eps", 0.0),
+])
+def test_bad_config_rejected_before_device_work(pkg, field, value):
+    cfg = pkg.make_config(synth.SO400M_224)
+    setattr(cfg, field, value)
+    assert pkg.ivit_weights_size(cfg) == 0
+    with pytest.raises(pkg.IvitError) as e:
+        pkg.ivit_create(cfg, np.zeros(8, np.uint16))
+    assert e.value.code == pkg.IVIT_ERR_SHAPE
+    assert pkg.ivit_last_error(None)
+
+
+def test_too_many_tokens_rejected(pkg):
+    cfg = pkg.make_config(synth.EncoderShape(896, 896, 14, 1152, 1, 16, 4304))  # 4096 tokens
+    with pytest.raises(pkg.IvitError) as e:
+        pkg.ivit_create(cfg, np.zeros(8, np.uint16))
+    assert "1024" in str(e.value)
+
+
+def test_null_handle_calls_return_arg_error(pkg):
+    L = pkg.load()
+    assert L.ivit_encode_full(None, None, None, None) == pkg.IVIT_ERR_ARG
+    assert L.ivit_encode_incremental(None, None, None, None, None) == pkg.IVIT_ERR_ARG
+    assert L.ivit_reset(None, 0) == pkg.IVIT_ERR_ARG
+    assert L.ivit_get_changed(None, 0, None, None, None) == pkg.IVIT_ERR_ARG
+    assert L.ivit_device_status(None, None) == pkg.IVIT_ERR_ARG
+    L.ivit_destroy(None)

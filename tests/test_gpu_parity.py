@@ -1,0 +1,127 @@
+"""GPU parity: the CUDA library through its C ABI against the oracle (small shapes that
+span several tiles and ragged tails, plus the edge cases of the method)."""
+import numpy as np
+import pytest
+
+from paper_2607_12287_gb300 import synth
+from tests.gpu_util import assert_tokens_close, run_side_by_side
+
+pytestmark = pytest.mark.gpu
+
+# D=320 (2.5 feature tiles), F=840 (6.6 tiles, ragged K for the MLP down projection),
+# P=14 (K=588, ragged), dh=64; 3 views of 64 tokens.
+SHAPE_A = synth.EncoderShape(112, 112, 14, 320, 2, 5, 840, synth.GELU_TANH)
+# N=196 tokens per view, D=192 (1.5 tiles), erf GELU; 2 streams x 1 view = 392 rows.
+SHAPE_B = synth.EncoderShape(224, 224, 16, 192, 2, 3, 768, synth.GELU_ERF)
+# dh=72 (SigLIP head width), F=1000.
+SHAPE_C = synth.EncoderShape(56, 56, 14, 576, 1, 8, 1000, synth.GELU_TANH)
+
+
+@pytest.fixture(scope="module")
+def pkg():
+    import paper_2607_12287_gb300 as p
+    p.load()
+    return p
+
+
+@pytest.mark.parametrize("shape,S,V", [(SHAPE_A, 1, 3), (SHAPE_B, 2, 1), (SHAPE_C, 1, 2)],
+                         ids=["A_d320_3view", "B_n196_2stream", "C_dh72"])
+def test_random_repaint_stream(pkg, oracle_mod, shape, S, V):
+    w = synth.make_weights(shape, 5)
+    frames = list(synth.stream_random(shape, S * V, 4, 6, change_p=0.2))
+    run_side_by_side(pkg, oracle_mod, shape, w, frames, S, V, check_caches=True)
+
+
+def test_identical_frames_select_nothing(pkg, oracle_mod):
+    import torch
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 7)
+    f0, f1 = synth.stream_random(shape, 2, 2, 8)
+    enc = pkg.IncrementalViT(shape, w, 1, 2)
+    d0, d1 = torch.from_numpy(f0).cuda(), torch.from_numpy(f1).cuda()
+    enc.encode_full(d0)
+    a, _ = enc.encode_incremental(d1)
+    b, counts = enc.encode_incremental(d1)  # same frame again: nothing to update
+    assert counts.cpu().tolist() == [0, 0]
+    assert torch.equal(a, b)
+    assert enc.device_status() == 0
+    enc.close()
+
+
+def test_single_token_and_mixed_views(pkg, oracle_mod):
+    # view 0 changes one patch, view 1 nothing, view 2 every patch
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 9)
+    rng = np.random.default_rng(10)
+    f0 = rng.integers(0, 256, (3, shape.img_h, shape.img_w, 3), dtype=np.uint8)
+    f1 = f0.copy()
+    f1[0, 14:28, 28:42] = rng.integers(0, 256, (14, 14, 3), dtype=np.uint8)
+    f1[2] = rng.integers(0, 256, f1[2].shape, dtype=np.uint8)
+    stats = run_side_by_side(pkg, oracle_mod, shape, w, [f0, f1, f1], 1, 3)
+    assert stats[1][2].tolist() == [1, 0, shape.n_tokens]
+    assert stats[2][2].tolist() == [0, 0, 0]
+
+
+def test_all_changed_incremental_matches_full(pkg, oracle_mod):
+    import torch
+    shape = SHAPE_B
+    w = synth.make_weights(shape, 11)
+    f0, f1 = synth.stream_random(shape, 2, 2, 12)
+    a = pkg.IncrementalViT(shape, w, 2, 1, threshold=2.0)  # every sim < 2
+    a.encode_full(torch.from_numpy(f0).cuda())
+    inc, counts = a.encode_incremental(torch.from_numpy(f1).cuda())
+    assert counts.cpu().tolist() == [shape.n_tokens] * 2
+    b = pkg.IncrementalViT(shape, w, 2, 1)
+    full = b.encode_full(torch.from_numpy(f1).cuda())
+    assert_tokens_close(inc.float().cpu().numpy(), full.float().cpu().numpy(), "inc vs full")
+    a.close()
+    b.close()
+
+
+def test_cold_start_and_reset(pkg, oracle_mod):
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 13)
+    frames = list(synth.stream_random(shape, 4, 3, 14, change_p=0.1))
+    # cold start: the first incremental call encodes everything
+    stats = run_side_by_side(pkg, oracle_mod, shape, w, frames, 2, 2, first_full=False)
+    assert stats[0][2].tolist() == [shape.n_tokens] * 4
+
+
+def test_reset_one_stream(pkg, oracle_mod):
+    import torch
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 15)
+    f0, f1 = synth.stream_random(shape, 4, 2, 16, change_p=0.1)
+    enc = pkg.IncrementalViT(shape, w, 2, 2)
+    orc = oracle_mod.Oracle(shape, w, 2, 2)
+    enc.encode_full(torch.from_numpy(f0).cuda())
+    orc.encode_full(f0)
+    enc.reset(1)
+    orc.reset(1)
+    out, counts = enc.encode_incremental(torch.from_numpy(f1).cuda())
+    ref, rc, _, _ = orc.encode_incremental(f1)
+    assert counts.cpu().tolist() == rc.tolist()
+    assert rc[2] == rc[3] == shape.n_tokens
+    assert_tokens_close(out.float().cpu().numpy(), ref, "after reset")
+    with pytest.raises(pkg.IvitError):
+        enc.reset(2)
+    enc.close()
+
+
+@pytest.mark.parametrize("k", [0, 1, 7, 64])
+def test_topk_selection(pkg, oracle_mod, k):
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 17)
+    frames = list(synth.stream_repaint(shape, 2, 3, 7, 18))
+    stats = run_side_by_side(pkg, oracle_mod, shape, w, frames, 1, 2,
+                             select_mode=synth.SEL_TOPK, topk=k)
+    for s in stats[1:]:
+        assert s[2].tolist() == [min(k, shape.n_tokens)] * 2
+
+
+def test_last_refresh_reference(pkg, oracle_mod):
+    shape = SHAPE_C
+    w = synth.make_weights(shape, 19)
+    frames = list(synth.stream_random(shape, 2, 4, 20, change_p=0.3))
+    run_side_by_side(pkg, oracle_mod, shape, w, frames, 1, 2,
+                     ref_mode=synth.REF_LAST_REFRESH, check_caches=True)
