@@ -1,0 +1,345 @@
+"""Benchmark: incremental ViT encode of a streaming camera feed on one GB300 (or N
+replicas under torchrun).
+
+A step is one ``ivit_encode_incremental`` call on the next frame of a seeded synthetic
+stream (the whole hot path: embed, score, select, gather, every block on the updated
+rows, final-token scatter).  Default workload: SigLIP-So400m-shaped encoder, 224x224
+frames (256 tokens), one camera, about 10% dynamic patches per frame.
+
+Printed JSON line (rank 0): frames/s of the incremental path with the frames already
+resident in HBM (``value``), ms per frame, the same library's full re-encode on the
+same frames and the speedup over it, the end-to-end number through the C ABI with host
+buffers (``e2e``), the GEMM kernel family's achieved HBM bandwidth against the measured
+peak (``roofline``), the oracle's CPU throughput (``cpu_baseline``) and the SM clocks
+sampled during the timed region.
+
+``--impl reference`` times the oracle (the plain CPU restatement the library is checked
+against) on the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2607_12287_gb300 import synth  # noqa: E402
+
+METRIC = "ms/frame and frames/s incremental ViT encode at 10% dynamic tokens; x vs full encode"
+DEFAULT_WORKLOAD = "so400m_224_1view"
+
+
+def describe(wl) -> dict:
+    s = wl.shape
+    return {
+        "workload": wl.name,
+        "encoder": (f"{s.img_h}x{s.img_w} px, patch {s.patch} ({s.n_tokens} tokens/view), dim {s.dim}, "
+                    f"{s.depth} layers, {s.heads} heads, MLP {s.mlp_dim}, pre-LN, "
+                    f"{'tanh' if s.gelu == 0 else 'erf'} GELU, seeded random-init bf16 weights"),
+        "views": wl.sv,
+        "selection": ("threshold sim<%.2f" % wl.threshold) if wl.select_mode == 0 else f"top-{wl.topk}",
+        "scene": wl.scene,
+    }
+
+
+def read_peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d.get("hbm_gbs"), "bf16_tflops": d.get("bf16_tflops"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
+
+
+def gemm_traffic_per_launch():
+    """DRAM bytes per GEMM launch from the committed ncu summary, or None when the
+    kernel source changed since that capture."""
+    summ = os.path.join(ROOT, "profiles", "gemm_tc_kernel_so400m_224_1view.md")
+    if not os.path.exists(summ):
+        return None
+    text = open(summ).read()
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    h = re.search(r"gemm_source_sha256:\s*([0-9a-f]{64})", text)
+    if not m or not h:
+        return None
+    src = open(os.path.join(ROOT, "paper_2607_12287_gb300", "csrc", "gemm.cu"), "rb").read()
+    if hashlib.sha256(src).hexdigest() != h.group(1):
+        return None
+    return float(m.group(1))
+
+
+class ClockSampler:
+    """Samples SM clocks and throttle reasons with nvidia-smi while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or not self.path or not os.path.exists(self.path):
+            return None
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, flags in rows for i, f in enumerate(flags) if f == "Active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "samples": len(rows), "reasons": reasons}
+
+
+def make_frames(wl, n: int):
+    return [np.ascontiguousarray(f) for f in wl.frames(n)]
+
+
+def cpu_baseline(wl, weights, frames, budget_s: float = 20.0) -> dict:
+    """The oracle as it stands, on this host's cores: an untimed full encode of frame 0,
+    then incremental frames timed until ``budget_s`` is spent (at least one)."""
+    import oracle
+    orc = oracle.Oracle.for_workload(wl, weights)
+    orc.encode_full(frames[0])
+    done, t0 = 0, time.perf_counter()
+    while done + 1 < len(frames):
+        orc.encode_incremental(frames[done + 1])
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    el = time.perf_counter() - t0
+    orc.close()
+    cores = len(os.sched_getaffinity(0))
+    return {"value": done * wl.sv / el, "unit": "frames/s", "cores": cores, "kind": "oracle",
+            "sample": (f"oracle incremental encode of frames 1..{done} of the {wl.name} stream after an "
+                       f"untimed full encode of frame 0 ({el:.1f} s, OpenMP over {cores} cores)")}
+
+
+def run_reference(args, wl, rank: int) -> None:
+    if rank != 0:
+        return
+    weights = synth.make_weights(wl.shape, 0)
+    frames = make_frames(wl, 1 + args.warmup + args.steps)
+    import oracle
+    orc = oracle.Oracle.for_workload(wl, weights)
+    orc.encode_full(frames[0])
+    for t in range(args.warmup):
+        orc.encode_incremental(frames[1 + t])
+    t0 = time.perf_counter()
+    for t in range(args.steps):
+        orc.encode_incremental(frames[1 + args.warmup + t])
+    el = time.perf_counter() - t0
+    orc.close()
+    fps = args.steps * wl.sv / el
+    cores = len(os.sched_getaffinity(0))
+    line = {
+        "impl": "reference", "metric": METRIC, "value": fps, "unit": "frames/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic", "config": describe(wl),
+        "cpu_baseline": {"value": fps, "unit": "frames/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{args.steps} incremental frames after a full encode and "
+                                   f"{args.warmup} warm-up frames, OpenMP over {cores} cores"},
+        "e2e": {"value": fps, "unit": "frames/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main() -> None:
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ivit", choices=["ivit", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.workload in synth.WORKLOADS:
+        wl = synth.WORKLOADS[args.workload]
+    elif args.workload.startswith("so400m_224_sweep_"):
+        wl = synth.sweep_workload(int(args.workload.rsplit("_", 1)[1].rstrip("pct")) / 100.0)
+    else:
+        ap.error(f"unknown workload {args.workload}")
+
+    if args.impl == "reference":
+        run_reference(args, wl, rank)
+        return
+
+    import torch
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+
+    import paper_2607_12287_gb300 as pkg
+    dev = torch.device("cuda", local_rank)
+    weights = synth.make_weights(wl.shape, 0)
+    n_frames = 1 + args.warmup + args.steps
+    frames = make_frames(wl, n_frames)
+    frames_dev = [torch.from_numpy(f).to(dev) for f in frames]
+    enc = pkg.IncrementalViT.for_workload(wl, weights)
+    stream = torch.cuda.current_stream(dev)
+    out = enc.tokens_buffer()
+    counts = torch.zeros((n_frames, wl.sv), dtype=torch.int32, device=dev)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    def timed(fn_step, label):
+        """Full encode of frame 0, warm-up frames, then K timed steps (CUDA events)."""
+        enc.encode_full(frames_dev[0], out)
+        for t in range(args.warmup):
+            fn_step(1 + t)
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for t in range(args.steps):
+            fn_step(1 + args.warmup + t)
+        e1.record(stream)
+        e1.synchronize()
+        ms = e0.elapsed_time(e1)
+        barrier()
+        if dist is not None:
+            m = torch.tensor([ms], device=dev)
+            dist.all_reduce(m, op=dist.ReduceOp.MAX)
+            ms = float(m.item())
+        return ms
+
+    def inc_step(t):
+        pkg.ivit_encode_incremental(enc.h, frames_dev[t], out, counts[t], stream)
+
+    def full_step(t):
+        pkg.ivit_encode_full(enc.h, frames_dev[t], out, stream)
+
+    peaks = read_peaks()
+    with ClockSampler(local_rank) as clk:
+        inc_ms = timed(inc_step, "incremental")
+    clocks = clk.summary()
+    launches_per_step = pkg.ivit_last_launch_count(enc.h)
+    changed = counts[1 + args.warmup:].float().sum(1).cpu().numpy()
+    full_ms = timed(full_step, "full")
+
+    # e2e: host frames (pinned) -> device, encode through the C ABI, tokens + counts -> host
+    host_in = [torch.from_numpy(f).pin_memory() for f in frames]
+    host_out = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    host_cnt = torch.empty(wl.sv, dtype=torch.int32).pin_memory()
+    dev_in = torch.empty_like(frames_dev[0])
+    cnt_dev = torch.empty(wl.sv, dtype=torch.int32, device=dev)
+
+    def e2e_step(t):
+        dev_in.copy_(host_in[t], non_blocking=True)
+        pkg.ivit_encode_incremental(enc.h, dev_in, out, cnt_dev, stream)
+        host_out.copy_(out, non_blocking=True)
+        host_cnt.copy_(cnt_dev, non_blocking=True)
+
+    e2e_ms = timed(e2e_step, "e2e")
+
+    # per-launch timing of the GEMM family (events around each launch, separate pass)
+    pkg.ivit_profile_enable(enc.h, True)
+    enc.encode_full(frames_dev[0], out)
+    pkg.ivit_profile_read(enc.h)
+    for t in range(args.steps):
+        inc_step(1 + args.warmup + t)
+    gemm_ms, gemm_n, gemm_bytes = pkg.ivit_profile_read(enc.h)
+    pkg.ivit_profile_enable(enc.h, False)
+    status = enc.device_status()
+
+    frames_total = args.steps * wl.sv * world
+    value = frames_total / (inc_ms / 1e3)
+    achieved = (gemm_bytes / gemm_n) / (gemm_ms / gemm_n / 1e3) / 1e9 if gemm_n else None
+    traffic = gemm_traffic_per_launch()
+    line = {
+        "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": inc_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": dict(describe(wl), **{
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+            "l2": "weights (%.0f MB bf16) are streamed every step: working set > 129 MB L2, no flush"
+                  % (synth.weight_count(wl.shape) * 2 / 1e6),
+            "changed_tokens_per_frame_mean": float(changed.mean()) / wl.sv,
+            "dynamic_fraction_mean": float(changed.mean()) / (wl.sv * wl.shape.n_tokens),
+        }),
+        "ms_per_frame": inc_ms / args.steps / wl.sv,
+        "full_encode_ms_per_step": full_ms / args.steps,
+        "full_encode_frames_per_s": frames_total / (full_ms / 1e3),
+        "speedup_vs_full": full_ms / inc_ms,
+        "e2e": {"value": frames_total / (e2e_ms / 1e3), "unit": "frames/s",
+                "ms_per_step": e2e_ms / args.steps,
+                "h2d_bytes_per_step": int(frames[0].nbytes),
+                "d2h_bytes_per_step": int(out.numel() * out.element_size() + wl.sv * 4)},
+        "roofline": {"kernel": "gemm_tc_kernel (all QKV/out-proj/MLP/embed launches)", "bound": "hbm",
+                     "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": (achieved / peaks["hbm_gbs"]) if achieved else None,
+                     "traffic": traffic, "peak_source": peaks["source"],
+                     "launches_timed": gemm_n, "avg_launch_us": 1e3 * gemm_ms / gemm_n if gemm_n else None,
+                     "algorithmic_bytes_per_launch": gemm_bytes / gemm_n if gemm_n else None},
+        "gpu_launches": int(launches_per_step * args.steps),
+        "launches_per_step": int(launches_per_step),
+        "device_status": status,
+        "clocks": clocks,
+    }
+    if rank == 0 and not args.no_cpu:
+        line["cpu_baseline"] = cpu_baseline(wl, weights, frames)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    enc.close()
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
