@@ -136,6 +136,33 @@ int64_t ivit_last_launch_count(const ivit_handle* h);
 
 void ivit_destroy(ivit_handle* h);
 
+/* Token selection that allocates nothing.  The paper has no counterpart: this entry
+ * point exists for callers that cannot call cudaMalloc when they need the lists --
+ * code enqueuing work while a stream is captured into a CUDA graph (allocation is not
+ * permitted there), plugins whose host framework forbids allocation inside its enqueue
+ * callback, and real-time loops that allocate only at start-up.
+ *
+ * It computes what the selection step of ivit_encode_incremental computes (cosine of
+ * each token against its reference in fp32, then threshold or top-k), from embeddings
+ * the caller holds: e_cur_dev and e_ref_dev fp32 [n_views][n_tok][dim].  Outputs, all
+ * caller-owned device memory: idx_out_dev int32 [n_views][n_tok] (ascending updated
+ * indices, then -1), counts_out_dev int32 [n_views].  Enqueued on `stream`; no handle.
+ *
+ * Its scratch (one fp32 score per token) is a file-scope device array of
+ * IVIT_NOALLOC_MAX_TOKENS floats (256 KiB) that every GPU loading the library holds
+ * until the process exits.  n_views * n_tok above that maximum returns IVIT_ERR_SHAPE
+ * (message via ivit_last_error(NULL)); no cudaMalloc, cudaFree or allocating library
+ * routine is ever called.  The first call on a device, with that device current, looks
+ * up the array's device address (cudaGetSymbolAddress) and caches it: make that first
+ * call before any stream capture.  All calls share the array; each call writes every
+ * score it reads, so nothing carries over, but calls that overlap on the GPU (two
+ * streams, or two threads) race on it and must be serialised by the caller. */
+#define IVIT_NOALLOC_MAX_TOKENS 65536
+int ivit_select_noalloc(const float* e_cur_dev, const float* e_ref_dev, int32_t n_views,
+                        int32_t n_tok, int32_t dim, int32_t select_mode, float threshold,
+                        int32_t topk, int32_t* idx_out_dev, int32_t* counts_out_dev,
+                        void* stream);
+
 /* Message of the last failure on `h` (or of the last failed create if h is NULL). */
 const char* ivit_last_error(const ivit_handle* h);
 

@@ -29,8 +29,9 @@ EXPORTED = [
     "ivit_weights_size", "ivit_create", "ivit_encode_full", "ivit_encode_incremental",
     "ivit_get_changed", "ivit_get_cache", "ivit_reset", "ivit_profile_enable",
     "ivit_profile_read", "ivit_device_status", "ivit_last_launch_count", "ivit_destroy",
-    "ivit_last_error",
+    "ivit_last_error", "ivit_select_noalloc",
 ]
+IVIT_NOALLOC_MAX_TOKENS = 65536
 
 
 class IvitConfig(C.Structure):
@@ -79,6 +80,8 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.ivit_destroy.restype = None
     L.ivit_last_error.restype = C.c_char_p
     L.ivit_last_error.argtypes = [P]
+    L.ivit_select_noalloc.argtypes = [P, P, C.c_int32, C.c_int32, C.c_int32, C.c_int32,
+                                      C.c_float, C.c_int32, P, P, P]
     _lib = L
     return L
 
@@ -175,6 +178,15 @@ def ivit_last_launch_count(h: int) -> int:
 
 def ivit_destroy(h: int) -> None:
     load().ivit_destroy(h)
+
+
+def ivit_select_noalloc(e_cur, e_ref, n_views: int, n_tok: int, dim: int, select_mode: int,
+                        threshold: float, topk: int, idx_out, counts_out, stream=None) -> None:
+    """Selection without device allocation (scratch in a fixed device array); for callers
+    that cannot allocate, e.g. while a stream is being captured into a CUDA graph."""
+    _check(load().ivit_select_noalloc(_ptr(e_cur), _ptr(e_ref), n_views, n_tok, dim, select_mode,
+                                      threshold, topk, _ptr(idx_out), _ptr(counts_out),
+                                      _stream(stream)), None)
 
 
 # ------------------------------------------------------------ convenience

@@ -1,6 +1,6 @@
 """Builds the CUDA library ``_build/libivit.so`` for sm_103a with nvcc.
 
-The three translation units compile in parallel; the shared object links the CUDA
+The translation units compile in parallel; the shared object links the CUDA
 runtime statically, so loading it needs no GPU and no driver library.
 """
 from __future__ import annotations
@@ -15,7 +15,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libivit.so")
-SOURCES = ["gemm.cu", "ops.cu", "engine.cu"]
+SOURCES = ["gemm.cu", "ops.cu", "engine.cu", "noalloc.cu"]
 HEADERS = ["ptx.cuh", "internal.h"]
 NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

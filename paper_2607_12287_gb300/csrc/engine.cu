@@ -84,6 +84,10 @@ inline float bf16_bits_to_float(uint16_t b) {
 
 }  // namespace
 
+namespace ivit {
+void set_create_error(const char* msg) { g_create_error = msg ? msg : ""; }
+}  // namespace ivit
+
 struct ivit_handle {
   ivit_config cfg{};
   int N = 0, D = 0, F = 0, H = 0, L = 0, SV = 0, Kp = 0, KPAD = 0, M_max = 0;
