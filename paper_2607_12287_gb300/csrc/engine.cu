@@ -7,7 +7,9 @@
 #include <cudaTypedefs.h>
 
 #include <cmath>
+#include <cstdlib>
 #include <cstdio>
+#include <algorithm>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -29,6 +31,13 @@ struct LayerW {
 struct EventPair {
   cudaEvent_t a, b;
 };
+
+// Launch shape of one GEMM: row-tile variant, CTAs per cluster (the K split), clusters.
+struct GemmPlan {
+  int bn = 64, csize = 1, n_clusters = 1;
+};
+
+enum GemmSlot { kGemmEmbed = 0, kGemmQKV, kGemmO, kGemmUp, kGemmDown, kGemmSlots };
 
 thread_local std::string g_create_error;
 
@@ -92,8 +101,8 @@ struct ivit_handle {
   ivit_config cfg{};
   int N = 0, D = 0, F = 0, H = 0, L = 0, SV = 0, Kp = 0, KPAD = 0, M_max = 0;
   int device = 0, num_sms = 0;
-  int grid64 = 0, grid256 = 0, row_grid = 0, bn_embed = 256, bn_inc = 64;
-  size_t ws_bytes = 0;
+  int row_grid = 0;
+  GemmPlan plan_full[kGemmSlots], plan_inc[kGemmSlots];
 
   void* wmem = nullptr;  // weights (device)
   void* smem = nullptr;  // state + workspaces (device)
@@ -103,14 +112,24 @@ struct ivit_handle {
   CUtensorMap tm_pe, tm_patches, tm_xn, tm_o, tm_h;
 
   bf16* patches = nullptr;
-  float *e_t = nullptr, *e_ref = nullptr, *sims = nullptr, *x = nullptr, *ws = nullptr;
+  float *e_t = nullptr, *e_ref = nullptr, *sims = nullptr, *x = nullptr;
   int *idx = nullptr, *counts = nullptr, *cu_rows = nullptr, *rowtok = nullptr, *done_ctr = nullptr;
-  int *tile_ctr = nullptr, *err = nullptr;
+  int* err = nullptr;
   bf16 *xn = nullptr, *q = nullptr, *o = nullptr, *hbuf = nullptr, *cacheK = nullptr,
        *cacheV = nullptr, *tok_out = nullptr;
 
   std::vector<uint8_t> cold;
   int64_t launches = 0;
+
+  // CUDA graphs of the full and the steady-state incremental chain.  Inputs and outputs
+  // are staged through handle-owned buffers (copies outside the graph), so the graph's
+  // kernel parameters never change.
+  bool use_graphs = true;
+  cudaStream_t cap_stream = nullptr;
+  cudaGraphExec_t graph_full = nullptr, graph_inc = nullptr;
+  int64_t graph_full_launches = 0, graph_inc_launches = 0;
+  uint8_t* frames_buf = nullptr;
+  int* counts_buf = nullptr;
 
   bool profiling = false;
   std::vector<EventPair> prof_events;
@@ -168,6 +187,31 @@ size_t weights_count(const ivit_config* c) {
   return D * Kp + D + N * D + per_layer * c->depth + 2 * D;
 }
 
+// Launch shape of a GEMM with a K split over clusters of c CTAs.  Cost model (fitted
+// to measurements of this kernel on GB300 with small row counts): a launch pays a fixed
+// ~4 us plus ~0.35 us per 16 KB weight stage a CTA streams, once per round of tiles
+// over the clusters that fit on the GPU.  Cluster sizes above 9 lose SMs to GPC packing.
+GemmPlan plan_gemm(int num_sms, int bn, int n_out, int k, int m_expected) {
+  GemmPlan best;
+  best.bn = bn;
+  const int n_ft = (n_out + 127) / 128, n_tt = (m_expected + bn - 1) / bn, n_kb = (k + 63) / 64;
+  const int tiles = std::max(1, n_ft * n_tt);
+  double best_cost = 1e30;
+  for (int c = 1; c <= std::min(16, n_kb); ++c) {
+    const int fit = ivit::gemm_max_clusters(bn, c);
+    if (fit <= 0) continue;
+    const int ncl = std::max(1, std::min({tiles, fit, num_sms / c}));
+    const int rounds = (tiles + ncl - 1) / ncl;
+    const double cost = rounds * (4.0 + 0.35 * ((n_kb + c - 1) / c));
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best.csize = c;
+      best.n_clusters = ncl;
+    }
+  }
+  return best;
+}
+
 int setup(ivit_handle* h, const uint16_t* wb) {
   const ivit_config& c = h->cfg;
   h->N = (c.img_h / c.patch) * (c.img_w / c.patch);
@@ -186,13 +230,32 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   IVIT_CK(h, cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device));
   IVIT_CK(h, ivit::gemm_setup(64));
   IVIT_CK(h, ivit::gemm_setup(256));
-  h->grid64 = h->num_sms * ivit::gemm_ctas_per_sm(64);
-  h->grid256 = h->num_sms * ivit::gemm_ctas_per_sm(256);
+  IVIT_CK(h, ivit::attention_setup());
+  if (std::getenv("IVIT_NO_PDL")) ivit::g_use_pdl = false;
+  if (std::getenv("IVIT_NO_GRAPH")) h->use_graphs = false;
+  IVIT_CK(h, cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking));
   h->row_grid = h->num_sms * 4;
-  h->bn_embed = M <= 64 ? 64 : 256;
-  h->bn_inc = M <= 1024 ? 64 : 256;
-  h->ws_bytes = std::max(static_cast<size_t>(h->grid64) * 64, static_cast<size_t>(h->grid256) * 256) *
-                128 * sizeof(float);
+  {
+    // Full encodes know M = SV*N.  Incremental calls are planned for a tenth of the
+    // tokens updated (any count still runs correctly, with more or fewer tile rounds).
+    const int m_inc = std::max(1, static_cast<int>(M / 10));
+    const int bn_full = M <= 64 ? 64 : 256, bn_inc = M <= 1024 ? 64 : 256;
+    const int shapes[kGemmSlots][2] = {{static_cast<int>(D), h->KPAD}, {3 * static_cast<int>(D), static_cast<int>(D)},
+                                       {static_cast<int>(D), static_cast<int>(D)}, {static_cast<int>(F), static_cast<int>(D)},
+                                       {static_cast<int>(D), static_cast<int>(F)}};
+    for (int g = 0; g < kGemmSlots; ++g) {
+      h->plan_full[g] = plan_gemm(h->num_sms, bn_full, shapes[g][0], shapes[g][1], static_cast<int>(M));
+      h->plan_inc[g] = g == kGemmEmbed ? h->plan_full[g]
+                                       : plan_gemm(h->num_sms, bn_inc, shapes[g][0], shapes[g][1], m_inc);
+    }
+    if (std::getenv("IVIT_DEBUG")) {
+      static const char* names[kGemmSlots] = {"embed", "qkv", "out", "up", "down"};
+      for (int g = 0; g < kGemmSlots; ++g)
+        std::fprintf(stderr, "ivit gemm %-5s full bn=%d cluster=%d x %d | inc bn=%d cluster=%d x %d\n",
+                     names[g], h->plan_full[g].bn, h->plan_full[g].csize, h->plan_full[g].n_clusters,
+                     h->plan_inc[g].bn, h->plan_inc[g].csize, h->plan_inc[g].n_clusters);
+    }
+  }
 
   // ---- weights: bf16 matrices (W_pe padded to KPAD columns), fp32 vectors
   Arena wa;
@@ -284,8 +347,9 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   const size_t o_x = sa.take(M * D * 4), o_xn = sa.take(M * D * 2), o_q = sa.take(M * D * 2);
   const size_t o_o = sa.take(M * D * 2), o_h = sa.take(M * F * 2);
   const size_t o_ck = sa.take(L * M * D * 2), o_cv = sa.take(L * M * D * 2), o_tok = sa.take(M * D * 2);
-  const size_t o_ws = sa.take(h->ws_bytes), o_tc = sa.take((h->grid64 + h->grid256) * 4);
   const size_t o_err = sa.take(4);
+  const size_t o_fb = sa.take(static_cast<size_t>(h->SV) * c.img_h * c.img_w * 3);
+  const size_t o_cb = sa.take(h->SV * 4);
   IVIT_CK(h, cudaMalloc(&h->smem, sa.size));
   IVIT_CK(h, cudaMemset(h->smem, 0, sa.size));
   sa.base = static_cast<char*>(h->smem);
@@ -306,9 +370,9 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   h->cacheK = sa.at<bf16>(o_ck);
   h->cacheV = sa.at<bf16>(o_cv);
   h->tok_out = sa.at<bf16>(o_tok);
-  h->ws = sa.at<float>(o_ws);
-  h->tile_ctr = sa.at<int>(o_tc);
   h->err = sa.at<int>(o_err);
+  h->frames_buf = sa.at<uint8_t>(o_fb);
+  h->counts_buf = sa.at<int>(o_cb);
   if (!make_map(&h->tm_patches, h->patches, h->KPAD, M, h->KPAD * 2, 64, 32) ||
       !make_map(&h->tm_xn, h->xn, D, M, D * 2, 64, 32) ||
       !make_map(&h->tm_o, h->o, D, M, D * 2, 64, 32) ||
@@ -319,6 +383,11 @@ int setup(ivit_handle* h, const uint16_t* wb) {
 }
 
 void release(ivit_handle* h) {
+  if (h->graph_full) cudaGraphExecDestroy(h->graph_full);
+  if (h->graph_inc) cudaGraphExecDestroy(h->graph_inc);
+  if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
+  h->graph_full = h->graph_inc = nullptr;
+  h->cap_stream = nullptr;
   if (h->wmem) cudaFree(h->wmem);
   if (h->smem) cudaFree(h->smem);
   for (auto& e : h->prof_events) {
@@ -335,14 +404,9 @@ double gemm_bytes(int n_out, int k, int kind, long long M) {
   return 2.0 * n_out * k + 2.0 * M * k + out_b * M * n_out + 4.0 * n_out;
 }
 
-int gemm(ivit_handle* h, int bn, const CUtensorMap& tw, const CUtensorMap& tx, ivit::GemmArgs a,
-         cudaStream_t s) {
+int gemm(ivit_handle* h, const GemmPlan& plan, const CUtensorMap& tw, const CUtensorMap& tx,
+         ivit::GemmArgs a, cudaStream_t s) {
   a.err = h->err;
-  a.tile_ctr = h->tile_ctr;
-  a.ws = h->ws;
-  a.ws_items = static_cast<int>(h->ws_bytes / (static_cast<size_t>(bn) * 128 * sizeof(float)));
-  a.max_splits = 16;
-  const int grid = bn == 64 ? h->grid64 : h->grid256;
   EventPair* ev = nullptr;
   if (h->profiling) {
     if (h->prof_used == h->prof_events.size()) {
@@ -354,7 +418,7 @@ int gemm(ivit_handle* h, int bn, const CUtensorMap& tw, const CUtensorMap& tx, i
     ev = &h->prof_events[h->prof_used++];
     IVIT_CK(h, cudaEventRecord(ev->a, s));
   }
-  IVIT_CK(h, ivit::launch_gemm(bn, tw, tx, a, grid, false, s));
+  IVIT_CK(h, ivit::launch_gemm(plan.bn, tw, tx, a, plan.n_clusters, plan.csize, s));
   ++h->launches;
   if (ev) {
     IVIT_CK(h, cudaEventRecord(ev->b, s));
@@ -366,15 +430,15 @@ int gemm(ivit_handle* h, int bn, const CUtensorMap& tw, const CUtensorMap& tx, i
   return IVIT_OK;
 }
 
-int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_counts, bool full,
-        cudaStream_t s) {
+// Enqueues the whole chain for one frame per view on `s` (eagerly or under capture).
+int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool full, cudaStream_t s) {
   const ivit_config& c = h->cfg;
   const int N = h->N, D = h->D, F = h->F, SV = h->SV, M = h->M_max;
   ivit::ColdMask cm;
   std::memset(&cm, 0, sizeof cm);
   for (int v = 0; v < SV; ++v)
     if (full || h->cold[v]) cm.bits[v >> 5] |= 1u << (v & 31);
-  const int bn = full ? 256 : h->bn_inc;
+  const GemmPlan* plan = full ? h->plan_full : h->plan_inc;
   const int* total = h->cu_rows + SV;
   h->launches = 0;
   h->call_static_bytes.clear();
@@ -390,7 +454,7 @@ int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_coun
     a.epi.bias = h->b_pe;
     a.epi.out_f32 = h->e_t;
     a.epi.ld_out = D;
-    if (int r = gemm(h, h->bn_embed, h->tm_pe, h->tm_patches, a, s)) return r;
+    if (int r = gemm(h, plan[kGemmEmbed], h->tm_pe, h->tm_patches, a, s)) return r;
   }
   if (!full) {
     IVIT_CK(h, ivit::launch_score(h->e_t, h->e_ref, h->sims, M, D, c.ref_mode == IVIT_REF_PREV_FRAME, s));
@@ -424,7 +488,7 @@ int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_coun
       a.epi.cache_v = cv;
       a.epi.rowtok = h->rowtok;
       a.epi.dim = D;
-      if (int r = gemm(h, bn, w.tm_qkv, h->tm_xn, a, s)) return r;
+      if (int r = gemm(h, plan[kGemmQKV], w.tm_qkv, h->tm_xn, a, s)) return r;
     }
     IVIT_CK(h, ivit::launch_attention(h->q, ck, cv, h->cu_rows, h->o, SV, N, D, h->H, s));
     ++h->launches;
@@ -437,7 +501,7 @@ int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_coun
       a.epi.bias = w.bo;
       a.epi.out_f32 = h->x;
       a.epi.ld_out = D;
-      if (int r = gemm(h, bn, w.tm_o, h->tm_o, a, s)) return r;
+      if (int r = gemm(h, plan[kGemmO], w.tm_o, h->tm_o, a, s)) return r;
     }
     IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln2g, w.ln2b, h->xn, nullptr, D, c.ln_eps, M,
                                       h->row_grid, s));
@@ -452,7 +516,7 @@ int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_coun
       a.epi.out_bf16 = h->hbuf;
       a.epi.ld_out = F;
       a.epi.gelu_mode = c.gelu;
-      if (int r = gemm(h, bn, w.tm_1, h->tm_xn, a, s)) return r;
+      if (int r = gemm(h, plan[kGemmUp], w.tm_1, h->tm_xn, a, s)) return r;
     }
     {
       ivit::GemmArgs a;
@@ -463,19 +527,59 @@ int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_coun
       a.epi.bias = w.b2;
       a.epi.out_f32 = h->x;
       a.epi.ld_out = D;
-      if (int r = gemm(h, bn, w.tm_2, h->tm_h, a, s)) return r;
+      if (int r = gemm(h, plan[kGemmDown], w.tm_2, h->tm_h, a, s)) return r;
     }
   }
   IVIT_CK(h, ivit::launch_layernorm(total, h->x, h->lnfg, h->lnfb, h->tok_out, h->rowtok, D, c.ln_eps,
                                     M, h->row_grid, s));
   ++h->launches;
-  if (out)
-    IVIT_CK(h, cudaMemcpyAsync(out, h->tok_out, static_cast<size_t>(M) * D * 2, cudaMemcpyDeviceToDevice, s));
+  return IVIT_OK;
+}
+
+int capture(ivit_handle* h, bool full, cudaGraphExec_t* exec, int64_t* launches) {
+  IVIT_CK(h, cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal));
+  const int r = run_core(h, h->frames_buf, h->counts_buf, full, h->cap_stream);
+  cudaGraph_t g = nullptr;
+  const cudaError_t e = cudaStreamEndCapture(h->cap_stream, &g);
+  if (r != IVIT_OK) {
+    if (g) cudaGraphDestroy(g);
+    return r;
+  }
+  if (e != cudaSuccess) return h->cuda_fail("cudaStreamEndCapture", e);
+  const cudaError_t ei = cudaGraphInstantiate(exec, g, 0);
+  cudaGraphDestroy(g);
+  if (ei != cudaSuccess) return h->cuda_fail("cudaGraphInstantiate", ei);
+  *launches = h->launches;
+  return IVIT_OK;
+}
+
+int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_counts, bool full,
+        cudaStream_t s) {
+  const int SV = h->SV;
+  const size_t tok_bytes = static_cast<size_t>(h->M_max) * h->D * 2;
+  bool any_cold = false;
+  for (int v = 0; v < SV; ++v) any_cold = any_cold || h->cold[v];
+  if (h->use_graphs && !h->profiling && (full || !any_cold)) {
+    cudaGraphExec_t* exec = full ? &h->graph_full : &h->graph_inc;
+    int64_t* nl = full ? &h->graph_full_launches : &h->graph_inc_launches;
+    if (!*exec)
+      if (int r = capture(h, full, exec, nl)) return r;
+    const size_t fbytes = static_cast<size_t>(SV) * h->cfg.img_h * h->cfg.img_w * 3;
+    IVIT_CK(h, cudaMemcpyAsync(h->frames_buf, frames, fbytes, cudaMemcpyDeviceToDevice, s));
+    IVIT_CK(h, cudaGraphLaunch(*exec, s));
+    if (out) IVIT_CK(h, cudaMemcpyAsync(out, h->tok_out, tok_bytes, cudaMemcpyDeviceToDevice, s));
+    if (user_counts && !full)
+      IVIT_CK(h, cudaMemcpyAsync(user_counts, h->counts_buf, SV * sizeof(int), cudaMemcpyDeviceToDevice, s));
+    h->launches = *nl;
+  } else {
+    if (int r = run_core(h, frames, user_counts, full, s)) return r;
+    if (out) IVIT_CK(h, cudaMemcpyAsync(out, h->tok_out, tok_bytes, cudaMemcpyDeviceToDevice, s));
+  }
   for (int v = 0; v < SV; ++v) h->cold[v] = 0;
 
   if (h->profiling) {
     int rows = 0;
-    IVIT_CK(h, cudaMemcpyAsync(&rows, total, sizeof(int), cudaMemcpyDeviceToHost, s));
+    IVIT_CK(h, cudaMemcpyAsync(&rows, h->cu_rows + SV, sizeof(int), cudaMemcpyDeviceToHost, s));
     IVIT_CK(h, cudaStreamSynchronize(s));
     for (size_t i = 0; i + 3 < h->call_static_bytes.size(); i += 4) {
       const double m = h->call_static_bytes[i + 3] >= 0 ? h->call_static_bytes[i + 3] : rows;

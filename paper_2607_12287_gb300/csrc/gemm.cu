@@ -5,14 +5,19 @@
 // output features) and the token rows are its B operand (N = 16..BN_MAX rows, rounded
 // up to 16), so a handful of updated tokens still fills the 128-row MMA: the kernel is
 // then a weight-streaming loop.  The row count M lives in device memory (written by the
-// selection kernel), so no host synchronisation is needed: every CTA reads M, derives
-// the same tiling (feature tiles x row tiles x K splits sized to the grid) and walks its
-// share of the work items.  K splits write fp32 partials; the last CTA to arrive on a
-// tile sums the partials in split order (deterministic) and runs the epilogue.
+// selection kernel), so no host synchronisation is needed: every CTA reads M and derives
+// the same tiling.
+//
+// The grid is a set of thread-block clusters.  The CTAs of a cluster split K of one
+// output tile between them (so many SMs stream one weight tile at once); each CTA
+// copies its fp32 partial tile from TMEM to its shared memory, and after a cluster
+// barrier every CTA sums a slice of the tile's rows over all CTAs' partials through
+// distributed shared memory, in rank order (deterministic), and runs the epilogue.
+// Clusters walk the output tiles (feature tile x row tile) with a stride.
 //
 // Pipeline per CTA (128 threads): warp 0 lane 0 issues TMA loads (weights with an
 // evict-first L2 policy, rows evict-last), warp 1 lane 0 issues tcgen05.mma into a TMEM
-// accumulator, all four warps run the epilogue from TMEM (tcgen05.ld, lane = feature).
+// accumulator, all four warps drain TMEM (tcgen05.ld, lane = output feature).
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -77,7 +82,7 @@ __global__ void __launch_bounds__(128, 1)
                                              ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR_OFFSET);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 1);
-  volatile int* sh_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);  // [0] last, [1] abort
+  volatile int* sh_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t smem_base = smem_u32(smem);
@@ -94,8 +99,7 @@ __global__ void __launch_bounds__(128, 1)
     fence_mbar_init();
     tma_prefetch_desc(&tm_w);
     tma_prefetch_desc(&tm_x);
-    sh_flag[0] = 0;
-    sh_flag[1] = 0;
+    *sh_abort = 0;
   }
   if (warp == 0) {
     tmem_alloc(smem_u32(tmem_slot), BN_MAX);
@@ -106,135 +110,168 @@ __global__ void __launch_bounds__(128, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  pdl_wait();  // outputs of the previous kernel on the stream are visible from here
-
+  const int csize = static_cast<int>(cluster_nctarank());
+  const int crank = static_cast<int>(cluster_ctarank());
+  const int cl_id = blockIdx.x / csize, n_cl = gridDim.x / csize;
+  // The row count comes from the selection kernel, at least two launches back: every
+  // kernel of the library triggers its dependents only after its own wait, so that
+  // kernel has completed by the time this grid can start.
   const int M = a.d_rows ? *a.d_rows : a.m_static;
   const int n_ft = (a.n_out + BM - 1) / BM;
   const int n_tt = (M + BN_MAX - 1) / BN_MAX;
   const int n_kb = (a.k + BK - 1) / BK;
-  const int base = n_ft * n_tt;
-  int splits = 1;
-  if (base > 0 && 2 * base <= static_cast<int>(gridDim.x)) {
-    splits = min(static_cast<int>(gridDim.x) / base, min(n_kb, a.max_splits));
-    if (splits * base > a.ws_items) splits = max(1, a.ws_items / base);
-  }
-  const int n_items = base * splits;
+  const int tiles = n_ft * n_tt;
+  const int kb0 = crank * n_kb / csize, kb1 = (crank + 1) * n_kb / csize;
+  const bool has_k = kb1 > kb0;
   const uint64_t pol_w = l2_policy_evict_first();
   const uint64_t pol_x = l2_policy_evict_last();
+  float* part = reinterpret_cast<float*>(smem);  // [rows][BM] fp32 partial (stage area)
+
+  // Weights do not depend on earlier kernels: start streaming the first tile's weight
+  // stages now, while the previous kernel may still be running.
+  int n_pre = 0;
+  if (warp == 0 && lane == 0 && cl_id < tiles && has_k) {
+    const int ft = cl_id % n_ft, tt = cl_id / n_ft;
+    const int n_mma = (min(BN_MAX, M - tt * BN_MAX) + 15) & ~15;
+    const int nbox = (n_mma + XBOX - 1) / XBOX;
+    n_pre = min(STAGES, kb1 - kb0);
+    for (int i = 0; i < n_pre; ++i) {
+      const uint32_t full = bar_base + 8 * i;
+      mbar_arrive_expect_tx(full, W_TILE_BYTES + nbox * XBOX_BYTES);
+      tma_load_2d(smem_base + i * L::STAGE_BYTES, &tm_w, (kb0 + i) * BK, ft * BM, full, pol_w);
+    }
+  }
+  pdl_wait();  // outputs of the previous kernel on the stream are visible from here
+  pdl_launch_dependents();
 
   uint32_t p_stage = 0, p_phase = 0;  // producer ring position
   uint32_t c_stage = 0, c_phase = 0;  // MMA ring position
   uint32_t acc_phase = 0;
 
-  for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
-    const int t = item % base, sp = item / base;
-    const int ft = t % n_ft, tt = t / n_ft;
-    const int kb0 = static_cast<int>(static_cast<long long>(sp) * n_kb / splits);
-    const int kb1 = static_cast<int>(static_cast<long long>(sp + 1) * n_kb / splits);
+  for (int tile = cl_id; tile < tiles; tile += n_cl) {
+    const int ft = tile % n_ft, tt = tile / n_ft;
     const int row0 = tt * BN_MAX;
     const int rows = min(BN_MAX, M - row0);
     const int n_mma = (rows + 15) & ~15;
     const int nbox = (n_mma + XBOX - 1) / XBOX;
+    bool ok = *sh_abort == 0;
 
-    if (warp == 0) {
-      if (lane == 0) {
-        for (int kb = kb0; kb < kb1; ++kb) {
-          const uint32_t empty = bar_base + 8 * (STAGES + p_stage);
-          const uint32_t full = bar_base + 8 * p_stage;
-          if (!mbar_wait(empty, p_phase ^ 1)) {
-            atomicExch(a.err, kErrWaitSlotEmpty);
-            sh_flag[1] = 1;
-            break;
-          }
-          const uint32_t st = smem_base + p_stage * L::STAGE_BYTES;
-          mbar_arrive_expect_tx(full, W_TILE_BYTES + nbox * XBOX_BYTES);
-          tma_load_2d(st, &tm_w, kb * BK, ft * BM, full, pol_w);
-          for (int b = 0; b < nbox; ++b)
-            tma_load_2d(st + W_TILE_BYTES + b * XBOX_BYTES, &tm_x, kb * BK, row0 + b * XBOX, full,
-                        pol_x);
-          if (++p_stage == STAGES) {
-            p_stage = 0;
-            p_phase ^= 1;
+    if (ok && has_k) {
+      if (warp == 0) {
+        if (lane == 0) {
+          const bool first = tile == cl_id;
+          for (int kb = kb0; kb < kb1; ++kb) {
+            const uint32_t empty = bar_base + 8 * (STAGES + p_stage);
+            const uint32_t full = bar_base + 8 * p_stage;
+            const uint32_t st = smem_base + p_stage * L::STAGE_BYTES;
+            if (!(first && kb - kb0 < n_pre)) {  // prefetched stages already hold the weights
+              if (!mbar_wait(empty, p_phase ^ 1)) {
+                atomicExch(a.err, kErrWaitSlotEmpty);
+                *sh_abort = 1;
+                break;
+              }
+              mbar_arrive_expect_tx(full, W_TILE_BYTES + nbox * XBOX_BYTES);
+              tma_load_2d(st, &tm_w, kb * BK, ft * BM, full, pol_w);
+            }
+            for (int b = 0; b < nbox; ++b)
+              tma_load_2d(st + W_TILE_BYTES + b * XBOX_BYTES, &tm_x, kb * BK, row0 + b * XBOX, full,
+                          pol_x);
+            if (++p_stage == STAGES) {
+              p_stage = 0;
+              p_phase ^= 1;
+            }
           }
         }
-      }
-      __syncwarp();
-    } else if (warp == 1) {
-      if (lane == 0) {
-        const uint32_t idesc = idesc_bf16_f32(BM, n_mma);
-        for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(bar_base + 8 * c_stage, c_phase)) {
-            atomicExch(a.err, kErrWaitTmaFull);
-            sh_flag[1] = 1;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t st = smem_base + c_stage * L::STAGE_BYTES;
+        __syncwarp();
+      } else if (warp == 1) {
+        if (lane == 0) {
+          const uint32_t idesc = idesc_bf16_f32(BM, n_mma);
+          for (int kb = kb0; kb < kb1; ++kb) {
+            if (!mbar_wait(bar_base + 8 * c_stage, c_phase)) {
+              atomicExch(a.err, kErrWaitTmaFull);
+              *sh_abort = 1;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t st = smem_base + c_stage * L::STAGE_BYTES;
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) {
-            const uint64_t ad = sdesc_kmajor_sw128(st + k * 32);
-            const uint64_t bd = sdesc_kmajor_sw128(st + W_TILE_BYTES + k * 32);
-            umma_bf16(tmem, ad, bd, idesc, (kb > kb0 || k > 0) ? 1u : 0u);
+            for (int k = 0; k < BK / 16; ++k) {
+              const uint64_t ad = sdesc_kmajor_sw128(st + k * 32);
+              const uint64_t bd = sdesc_kmajor_sw128(st + W_TILE_BYTES + k * 32);
+              umma_bf16(tmem, ad, bd, idesc, (kb > kb0 || k > 0) ? 1u : 0u);
+            }
+            umma_commit(bar_base + 8 * (STAGES + c_stage));  // frees the stage when read
+            if (++c_stage == STAGES) {
+              c_stage = 0;
+              c_phase ^= 1;
+            }
           }
-          umma_commit(bar_base + 8 * (STAGES + c_stage));  // frees the stage when read
-          if (++c_stage == STAGES) {
-            c_stage = 0;
-            c_phase ^= 1;
-          }
+          umma_commit(acc_bar);  // accumulator complete
         }
-        umma_commit(acc_bar);  // accumulator complete
+        __syncwarp();
       }
-      __syncwarp();
+      if (!mbar_wait(acc_bar, acc_phase)) {
+        atomicExch(a.err, kErrWaitAccum);
+        *sh_abort = 1;
+      }
+      acc_phase ^= 1;
     }
-
-    if (!mbar_wait(acc_bar, acc_phase)) {
-      atomicExch(a.err, kErrWaitAccum);
-      sh_flag[1] = 1;
-    }
-    acc_phase ^= 1;
     tc_fence_after();
     __syncthreads();
-    if (sh_flag[1]) break;
+    ok = *sh_abort == 0;
 
     const int fl = warp * 32 + lane;  // TMEM lane == tile-local output feature
-    const int f = ft * BM + fl;
     const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    if (splits == 1) {
-      for (int c0 = 0; c0 < rows; c0 += 16) {
-        float v[16];
-        tmem_ld16(trow + c0, v);
-        if (f < a.n_out) {
+    if (csize == 1) {
+      const int f = ft * BM + fl;
+      if (ok && has_k) {
+        for (int c0 = 0; c0 < rows; c0 += 16) {
+          float v[16];
+          tmem_ld16(trow + c0, v);
+          if (f < a.n_out) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            if (c0 + j < rows) epilogue_store(a.epi, row0 + c0 + j, f, v[j]);
+            for (int j = 0; j < 16; ++j)
+              if (c0 + j < rows) epilogue_store(a.epi, row0 + c0 + j, f, v[j]);
+          }
         }
       }
     } else {
-      float* part = a.ws + static_cast<size_t>(item) * (BN_MAX * BM);
-      for (int c0 = 0; c0 < rows; c0 += 16) {
-        float v[16];
-        tmem_ld16(trow + c0, v);
+      if (ok) {
+        if (has_k) {
+          for (int c0 = 0; c0 < rows; c0 += 16) {
+            float v[16];
+            tmem_ld16(trow + c0, v);
 #pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (c0 + j < rows) __stcg(part + (c0 + j) * BM + fl, v[j]);
-      }
-      __threadfence();
-      __syncthreads();
-      if (tid == 0) {
-        const int prev = atomicAdd(&a.tile_ctr[t], 1);
-        sh_flag[0] = (prev == splits - 1) ? 1 : 0;
-      }
-      __syncthreads();
-      if (sh_flag[0]) {
-        __threadfence();
-        for (int c = 0; c < rows; ++c) {
-          float acc = 0.f;
-          for (int s2 = 0; s2 < splits; ++s2)
-            acc += __ldcg(a.ws + static_cast<size_t>(s2 * base + t) * (BN_MAX * BM) + c * BM + fl);
-          if (f < a.n_out) epilogue_store(a.epi, row0 + c, f, acc);
+            for (int j = 0; j < 16; ++j)
+              if (c0 + j < rows) part[(c0 + j) * BM + fl] = v[j];
+          }
+        } else {
+          for (int c = 0; c < rows; ++c) part[c * BM + fl] = 0.f;
         }
-        if (tid == 0) a.tile_ctr[t] = 0;  // ready for the next launch
       }
+      cluster_sync();  // every partial of this tile is in its CTA's shared memory
+      if (ok) {
+        // this CTA's slice of the tile's rows; lane owns 4 consecutive features
+        const int c_lo = crank * rows / csize, c_hi = (crank + 1) * rows / csize;
+        const int f4 = ft * BM + 4 * lane;
+        const uint32_t part_addr = smem_u32(part);
+        for (int c = c_lo + warp; c < c_hi; c += 4) {
+          const uint32_t off = part_addr + static_cast<uint32_t>((c * BM + 4 * lane) * 4);
+          float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+          for (int s = 0; s < csize; ++s) {
+            const float4 p = ld_dsmem_f32x4(mapa_shared(off, s));
+            acc.x += p.x;
+            acc.y += p.y;
+            acc.z += p.z;
+            acc.w += p.w;
+          }
+          const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (f4 + j < a.n_out) epilogue_store(a.epi, row0 + c, f4 + j, vals[j]);
+        }
+      }
+      cluster_sync();  // partials stay valid until every CTA has read them
     }
     tc_fence_before();
     __syncthreads();
@@ -249,18 +286,52 @@ __global__ void __launch_bounds__(128, 1)
 
 template <int BN>
 cudaError_t launch_variant(const CUtensorMap& tm_w, const CUtensorMap& tm_x, const GemmArgs& a,
-                           int grid, bool pdl, cudaStream_t s) {
+                           int n_clusters, int csize, cudaStream_t s) {
+  // cluster dims are always given (also for a single CTA) so %cluster_nctarank is exact
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = dim3(n_clusters * csize);
   cfg.blockDim = dim3(128);
   cfg.dynamicSmemBytes = GemmSmem<BN>::TOTAL;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = csize;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = g_use_pdl ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<BN>, tm_w, tm_x, a);
+}
+
+template <int BN>
+int max_clusters_variant(int csize) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(csize);
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = GemmSmem<BN>::TOTAL;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = csize;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<BN>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+template <int BN>
+cudaError_t setup_variant() {
+  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       GemmSmem<BN>::TOTAL);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(gemm_tc_kernel<BN>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
 
 }  // namespace
@@ -269,29 +340,16 @@ size_t gemm_smem_bytes(int bn_max) {
   return bn_max == 64 ? GemmSmem<64>::TOTAL : GemmSmem<256>::TOTAL;
 }
 
-cudaError_t gemm_setup(int bn_max) {
-  if (bn_max == 64)
-    return cudaFuncSetAttribute(gemm_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                GemmSmem<64>::TOTAL);
-  return cudaFuncSetAttribute(gemm_tc_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              GemmSmem<256>::TOTAL);
-}
+cudaError_t gemm_setup(int bn_max) { return bn_max == 64 ? setup_variant<64>() : setup_variant<256>(); }
 
-int gemm_ctas_per_sm(int bn_max) {
-  int n = 0;
-  cudaError_t e;
-  if (bn_max == 64)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemm_tc_kernel<64>, 128, GemmSmem<64>::TOTAL);
-  else
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemm_tc_kernel<256>, 128,
-                                                      GemmSmem<256>::TOTAL);
-  return e == cudaSuccess && n > 0 ? n : 1;
+int gemm_max_clusters(int bn_max, int csize) {
+  return bn_max == 64 ? max_clusters_variant<64>(csize) : max_clusters_variant<256>(csize);
 }
 
 cudaError_t launch_gemm(int bn_max, const CUtensorMap& tm_w, const CUtensorMap& tm_x,
-                        const GemmArgs& a, int grid, bool pdl, cudaStream_t s) {
-  if (bn_max == 64) return launch_variant<64>(tm_w, tm_x, a, grid, pdl, s);
-  return launch_variant<256>(tm_w, tm_x, a, grid, pdl, s);
+                        const GemmArgs& a, int n_clusters, int csize, cudaStream_t s) {
+  if (bn_max == 64) return launch_variant<64>(tm_w, tm_x, a, n_clusters, csize, s);
+  return launch_variant<256>(tm_w, tm_x, a, n_clusters, csize, s);
 }
 
 }  // namespace ivit

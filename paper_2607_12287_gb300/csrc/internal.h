@@ -10,6 +10,38 @@ namespace ivit {
 
 using bf16 = __nv_bfloat16;
 
+// Programmatic dependent launch for every kernel of the library (on by default; the
+// IVIT_NO_PDL environment variable turns it off at handle creation).
+extern bool g_use_pdl;
+
+// cudaLaunchKernelEx with optional cluster width and the PDL attribute.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                      unsigned cluster_x, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  unsigned n = 0;
+  if (cluster_x > 1) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = cluster_x;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  if (g_use_pdl) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
+
 // ------------------------------------------------------------------ GEMM (tcgen05)
 // Y[r][f] = sum_k X[r][k] * W[f][k] for r < M rows, f < Nout features, then an
 // epilogue.  W is the weight matrix in Linear layout [Nout][K] (bf16, K-major), X the
@@ -40,22 +72,20 @@ struct GemmArgs {
   int k = 0;                     // K
   const int* d_rows = nullptr;   // device row count M (nullptr: use m_static)
   int m_static = 0;
-  int max_splits = 16;
-  float* ws = nullptr;           // split-K partials, ws_items x (bn_max x 128) fp32
-  int ws_items = 0;
-  int* tile_ctr = nullptr;       // one arrival counter per output tile, zero between launches
   int* err = nullptr;            // device error word
   GemmEpilogue epi;
 };
 
 // Returns the dynamic shared memory size (bytes) of the GEMM variant.
 size_t gemm_smem_bytes(int bn_max);
-// One-time attribute setup (dynamic smem opt-in).  Returns a CUDA error.
+// One-time attribute setup (dynamic smem opt-in, clusters of up to 16).
 cudaError_t gemm_setup(int bn_max);
-// Occupancy of the variant (CTAs per SM).
-int gemm_ctas_per_sm(int bn_max);
+// Clusters of `csize` CTAs of the variant that can be resident at once (0 if none).
+int gemm_max_clusters(int bn_max, int csize);
+// Launches n_clusters clusters of csize CTAs.  The CTAs of a cluster split K and reduce
+// their partial tiles through distributed shared memory; clusters walk the output tiles.
 cudaError_t launch_gemm(int bn_max, const CUtensorMap& tm_w, const CUtensorMap& tm_x,
-                        const GemmArgs& a, int grid, bool pdl, cudaStream_t s);
+                        const GemmArgs& a, int n_clusters, int csize, cudaStream_t s);
 
 // ------------------------------------------------------------------- other kernels
 struct ColdMask {
@@ -82,6 +112,9 @@ cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const flo
 cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma, const float* beta,
                              bf16* y, const int* dst_rowtok, int dim, float eps, int max_rows,
                              int grid, cudaStream_t s);
+
+// One-time function attributes of the attention kernel (dynamic shared memory opt-in).
+cudaError_t attention_setup();
 
 // O[r] = softmax(Q[r] K_v^T / sqrt(dh)) V_v per head, for the packed query rows r of
 // each view v (cu_rows), over the N cached keys/values of that view.

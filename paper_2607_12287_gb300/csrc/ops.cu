@@ -5,6 +5,9 @@
 #include "ptx.cuh"
 
 namespace ivit {
+
+bool g_use_pdl = true;
+
 namespace {
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -30,6 +33,7 @@ __device__ __forceinline__ bool is_cold(const ColdMask& m, int v) {
 __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __restrict__ patches,
                                 int sv, int img_h, int img_w, int P, int kpad) {
   pdl_wait();
+  pdl_launch_dependents();
   const int gw = img_w / P, gh = img_h / P, N = gw * gh;
   const long long total = static_cast<long long>(sv) * N * P;
   for (long long g = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; g < total;
@@ -52,6 +56,7 @@ __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __rest
 __global__ void score_kernel(const float* __restrict__ e_t, float* __restrict__ e_ref,
                              float* __restrict__ sims, int rows, int dim, int copy_ref) {
   pdl_wait();
+  pdl_launch_dependents();
   const int warps = blockDim.x >> 5;
   const int lane = threadIdx.x & 31;
   for (int r = blockIdx.x * warps + (threadIdx.x >> 5); r < rows; r += gridDim.x * warps) {
@@ -84,6 +89,7 @@ __global__ void select_kernel(const float* __restrict__ sims, int N, int sv, int
                               int* __restrict__ rowtok, int* __restrict__ done_ctr,
                               int* __restrict__ user_counts) {
   pdl_wait();
+  pdl_launch_dependents();
   extern __shared__ float s_sims[];  // [N]
   __shared__ int s_warp[32];
   __shared__ int s_last;
@@ -167,6 +173,7 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
                               float* __restrict__ x, float* __restrict__ e_ref, int N, int dim,
                               int ref_last_refresh, const ColdMask cold) {
   pdl_wait();
+  pdl_launch_dependents();
   const int rows = *total_rows;
   const int warps = blockDim.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -187,75 +194,108 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
 }
 
 // -------------------------------------------------------------------- layernorm
-// One warp per row; mean, then centred second moment, then the normalised output, in
-// fp32 (the row stays in L1 between passes).
+// One warp per row.  The row (up to 2048 floats) is read once into registers with
+// 128-bit loads; mean, centred second moment and the normalised output are computed
+// from registers in fp32.
+constexpr int LN_MAX_F4_PER_LANE = 16;
+
 __global__ void layernorm_kernel(const int* __restrict__ nrows, const float* __restrict__ x,
                                  const float* __restrict__ gamma, const float* __restrict__ beta,
                                  bf16* __restrict__ y, const int* __restrict__ dst_rowtok, int dim,
                                  float eps) {
   pdl_wait();
+  pdl_launch_dependents();
   const int rows = *nrows;
   const int warps = blockDim.x >> 5;
   const int lane = threadIdx.x & 31;
   const int n4 = dim / 4;
+  const float4* g4 = reinterpret_cast<const float4*>(gamma);
+  const float4* b4 = reinterpret_cast<const float4*>(beta);
   for (int r = blockIdx.x * warps + (threadIdx.x >> 5); r < rows; r += gridDim.x * warps) {
     const float4* xr = reinterpret_cast<const float4*>(x + static_cast<size_t>(r) * dim);
+    float4 v[LN_MAX_F4_PER_LANE];
     float sum = 0.f;
-    for (int c = lane; c < n4; c += 32) {
-      const float4 u = xr[c];
-      sum += (u.x + u.y) + (u.z + u.w);
+#pragma unroll
+    for (int i = 0; i < LN_MAX_F4_PER_LANE; ++i) {
+      const int c = lane + 32 * i;
+      v[i] = c < n4 ? xr[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+      sum += (v[i].x + v[i].y) + (v[i].z + v[i].w);
     }
     const float mean = warp_sum(sum) / dim;
     float sq = 0.f;
-    for (int c = lane; c < n4; c += 32) {
-      const float4 u = xr[c];
-      const float a = u.x - mean, b = u.y - mean, cc = u.z - mean, d = u.w - mean;
-      sq += (a * a + b * b) + (cc * cc + d * d);
+#pragma unroll
+    for (int i = 0; i < LN_MAX_F4_PER_LANE; ++i) {
+      if (lane + 32 * i < n4) {
+        const float a = v[i].x - mean, b = v[i].y - mean, c = v[i].z - mean, d = v[i].w - mean;
+        sq += (a * a + b * b) + (c * c + d * d);
+      }
     }
     const float rstd = rsqrtf(warp_sum(sq) / dim + eps);
     const size_t orow = dst_rowtok ? static_cast<size_t>(dst_rowtok[r]) : static_cast<size_t>(r);
     __nv_bfloat162* yr = reinterpret_cast<__nv_bfloat162*>(y + orow * dim);
-    const float4* g4 = reinterpret_cast<const float4*>(gamma);
-    const float4* b4 = reinterpret_cast<const float4*>(beta);
-    for (int c = lane; c < n4; c += 32) {
-      const float4 u = xr[c], g = g4[c], b = b4[c];
-      yr[2 * c] = __floats2bfloat162_rn(g.x * (u.x - mean) * rstd + b.x, g.y * (u.y - mean) * rstd + b.y);
-      yr[2 * c + 1] = __floats2bfloat162_rn(g.z * (u.z - mean) * rstd + b.z, g.w * (u.w - mean) * rstd + b.w);
+#pragma unroll
+    for (int i = 0; i < LN_MAX_F4_PER_LANE; ++i) {
+      const int c = lane + 32 * i;
+      if (c < n4) {
+        const float4 g = g4[c], b = b4[c], u = v[i];
+        yr[2 * c] = __floats2bfloat162_rn(g.x * (u.x - mean) * rstd + b.x, g.y * (u.y - mean) * rstd + b.y);
+        yr[2 * c + 1] = __floats2bfloat162_rn(g.z * (u.z - mean) * rstd + b.z, g.w * (u.w - mean) * rstd + b.w);
+      }
     }
   }
 }
 
 // -------------------------------------------------------------------- attention
-// CTA = (query block of one view, head).  Keys and values of the view are streamed in
-// tiles of KT rows through shared memory (fp32, padded rows); each warp owns QPW
-// queries and keeps an online softmax (running max and sum) and its output row in
-// registers: lane d owns output dims d, d+32, d+64, d+96.
-constexpr int ATT_WARPS = 4;
-constexpr int ATT_QPW = 8;
+// Attention of the updated queries of one view over all N keys of that view (cached
+// K/V with this call's updated rows already written), per head:
+//   O = softmax(Q K^T / sqrt(dh)) V.
+// Grid: (query block x key split, head, view); the key splits of one query block form
+// a thread-block cluster.  Each CTA streams its key range in tiles of ATT_KT through
+// shared memory (16-byte loads; K stored transposed so lanes read consecutive keys),
+// keeps an online softmax per query (running max m, sum l, output row in registers),
+// then the cluster merges its partial (m, l, o) through distributed shared memory:
+//   M = max_s m_s,  O = sum_s exp(m_s - M) o_s / sum_s exp(m_s - M) l_s.
+// Warp w owns queries 4w..4w+3 of the block; lane owns keys lane, lane+32 of a tile
+// for the scores and output dims lane + 32c for P V.
+constexpr int ATT_WARPS = 8;
+constexpr int ATT_QPW = 4;
 constexpr int ATT_QB = ATT_WARPS * ATT_QPW;
 constexpr int ATT_KT = 64;
 
 __global__ void __launch_bounds__(ATT_WARPS * 32)
     attention_kernel(const bf16* __restrict__ q, const bf16* __restrict__ cache_k,
                      const bf16* __restrict__ cache_v, const int* __restrict__ cu_rows,
-                     bf16* __restrict__ o, int N, int dim, int dh) {
+                     bf16* __restrict__ o, int N, int dim, int dh, int keys_per_split) {
   pdl_wait();
+  pdl_launch_dependents();
   extern __shared__ float sm[];
-  const int ld = dh + 1;
-  float* sk = sm;                       // [KT][dh+1]
-  float* sv = sk + ATT_KT * ld;         // [KT][dh+1]
-  float* sq = sv + ATT_KT * ld;         // [QB][dh]
-  const int v = blockIdx.z, h = blockIdx.y;
+  float* skT = sm;                          // [dh][KT]   (after the key loop: partial o [QB][dh])
+  float* sv = skT + dh * ATT_KT;            // [KT][dh]
+  float* sq = sv + ATT_KT * dh;             // [QB][dh]
+  float* sp = sq + ATT_QB * dh;             // [WARPS][QPW][KT]
+  float* sml = sp + ATT_WARPS * ATT_QPW * ATT_KT;  // [QB][2]
+  const int ns = static_cast<int>(cluster_nctarank());
+  const int rank = static_cast<int>(cluster_ctarank());
+  const int v = blockIdx.z, h = blockIdx.y, qb = blockIdx.x / ns;
   const int r_begin = cu_rows[v], r_end = cu_rows[v + 1];
-  const int q0 = r_begin + blockIdx.x * ATT_QB;
-  if (q0 >= r_end) return;
+  const int q0 = r_begin + qb * ATT_QB;
+  if (q0 >= r_end) return;  // the whole cluster shares qb, so it leaves together
   const int nq = min(ATT_QB, r_end - q0);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int dh8 = dh / 8;
   const float scale = rsqrtf(static_cast<float>(dh));
+  const int k_begin = rank * keys_per_split, k_end = min(N, k_begin + keys_per_split);
 
-  for (int e = tid; e < nq * dh; e += blockDim.x) {
-    const int qi = e / dh, d = e % dh;
-    sq[qi * dh + d] = __bfloat162float(q[static_cast<size_t>(q0 + qi) * dim + h * dh + d]) * scale;
+  for (int e = tid; e < nq * dh8; e += blockDim.x) {
+    const int qi = e / dh8, c = e % dh8;
+    const uint4 u = *reinterpret_cast<const uint4*>(q + static_cast<size_t>(q0 + qi) * dim + h * dh + c * 8);
+    const __nv_bfloat162* b2 = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(b2[i]);
+      sq[qi * dh + c * 8 + 2 * i] = f.x * scale;
+      sq[qi * dh + c * 8 + 2 * i + 1] = f.y * scale;
+    }
   }
 
   float m_run[ATT_QPW], l_run[ATT_QPW], acc[ATT_QPW][4];
@@ -266,66 +306,134 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc[a][c] = 0.f;
   }
-
   const size_t vbase = static_cast<size_t>(v) * N;
-  for (int k0 = 0; k0 < N; k0 += ATT_KT) {
-    const int nk = min(ATT_KT, N - k0);
+  float* spw = sp + warp * ATT_QPW * ATT_KT;
+
+  for (int k0 = k_begin; k0 < k_end; k0 += ATT_KT) {
+    const int nk = min(ATT_KT, k_end - k0);
     __syncthreads();
-    for (int e = tid; e < nk * dh; e += blockDim.x) {
-      const int j = e / dh, d = e % dh;
-      const size_t g = (vbase + k0 + j) * dim + h * dh + d;
-      sk[j * ld + d] = __bfloat162float(cache_k[g]);
-      sv[j * ld + d] = __bfloat162float(cache_v[g]);
+    for (int e = tid; e < ATT_KT * dh8; e += blockDim.x) {
+      const int j = e % ATT_KT, c = e / ATT_KT;
+      if (j < nk) {
+        const size_t g = (vbase + k0 + j) * dim + h * dh + c * 8;
+        const uint4 uk = *reinterpret_cast<const uint4*>(cache_k + g);
+        const uint4 uv = *reinterpret_cast<const uint4*>(cache_v + g);
+        const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&uk);
+        const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&uv);
+        float4* vd = reinterpret_cast<float4*>(sv + j * dh + c * 8);
+        float tv[8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 fk = __bfloat1622float2(k2[i]);
+          skT[(c * 8 + 2 * i) * ATT_KT + j] = fk.x;
+          skT[(c * 8 + 2 * i + 1) * ATT_KT + j] = fk.y;
+          const float2 fv = __bfloat1622float2(v2[i]);
+          tv[2 * i] = fv.x;
+          tv[2 * i + 1] = fv.y;
+        }
+        vd[0] = make_float4(tv[0], tv[1], tv[2], tv[3]);
+        vd[1] = make_float4(tv[4], tv[5], tv[6], tv[7]);
+      }
     }
     __syncthreads();
+
+    // scores of this warp's queries against the tile (lane: keys lane and lane + 32)
+    float s0[ATT_QPW], s1[ATT_QPW];
+#pragma unroll
+    for (int a = 0; a < ATT_QPW; ++a) s0[a] = s1[a] = 0.f;
+    const float* qw = sq + warp * ATT_QPW * dh;
+    for (int d = 0; d < dh; ++d) {
+      const float k0v = skT[d * ATT_KT + lane], k1v = skT[d * ATT_KT + lane + 32];
+#pragma unroll
+      for (int a = 0; a < ATT_QPW; ++a) {
+        const float qv = qw[a * dh + d];
+        s0[a] += qv * k0v;
+        s1[a] += qv * k1v;
+      }
+    }
 #pragma unroll
     for (int a = 0; a < ATT_QPW; ++a) {
-      const int qi = warp * ATT_QPW + a;
-      if (qi >= nq) break;
-      const float* qr = sq + qi * dh;
-      float s0 = -INFINITY, s1 = -INFINITY;
-      if (lane < nk) {
-        float t = 0.f;
-        for (int d = 0; d < dh; ++d) t += qr[d] * sk[lane * ld + d];
-        s0 = t;
-      }
-      if (lane + 32 < nk) {
-        float t = 0.f;
-        for (int d = 0; d < dh; ++d) t += qr[d] * sk[(lane + 32) * ld + d];
-        s1 = t;
-      }
-      const float mt = warp_max(fmaxf(s0, s1));
-      const float m_new = fmaxf(m_run[a], mt);
+      const float x0 = lane < nk ? s0[a] : -INFINITY;
+      const float x1 = lane + 32 < nk ? s1[a] : -INFINITY;
+      const float m_new = fmaxf(m_run[a], warp_max(fmaxf(x0, x1)));
       const float corr = __expf(m_run[a] - m_new);
-      const float p0 = (lane < nk) ? __expf(s0 - m_new) : 0.f;
-      const float p1 = (lane + 32 < nk) ? __expf(s1 - m_new) : 0.f;
+      const float p0 = lane < nk ? __expf(x0 - m_new) : 0.f;
+      const float p1 = lane + 32 < nk ? __expf(x1 - m_new) : 0.f;
       l_run[a] = l_run[a] * corr + warp_sum(p0 + p1);
       m_run[a] = m_new;
 #pragma unroll
       for (int c = 0; c < 4; ++c) acc[a][c] *= corr;
-      for (int j = 0; j < nk; ++j) {
-        const float pj = __shfl_sync(0xffffffffu, j < 32 ? p0 : p1, j & 31);
-        const float* vr = sv + j * ld;
+      spw[a * ATT_KT + lane] = p0;
+      spw[a * ATT_KT + lane + 32] = p1;
+    }
+    __syncwarp();
+    for (int j = 0; j < nk; ++j) {
+      float vv[4];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const int d = lane + 32 * c;
-          if (d < dh) acc[a][c] += pj * vr[d];
-        }
+      for (int c = 0; c < 4; ++c) vv[c] = (lane + 32 * c < dh) ? sv[j * dh + lane + 32 * c] : 0.f;
+#pragma unroll
+      for (int a = 0; a < ATT_QPW; ++a) {
+        const float pj = spw[a * ATT_KT + j];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[a][c] += pj * vv[c];
       }
     }
+    __syncwarp();
   }
+
+  if (ns == 1) {
+#pragma unroll
+    for (int a = 0; a < ATT_QPW; ++a) {
+      const int qi = warp * ATT_QPW + a;
+      if (qi < nq) {
+        const float inv = 1.f / l_run[a];
+        bf16* orow = o + static_cast<size_t>(q0 + qi) * dim + h * dh;
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+          if (lane + 32 * c < dh) orow[lane + 32 * c] = __float2bfloat16_rn(acc[a][c] * inv);
+      }
+    }
+    return;
+  }
+
+  // partial (m, l, o) of every query of the block, then a cluster-wide merge
+  __syncthreads();
+  float* so = skT;  // [QB][dh]
 #pragma unroll
   for (int a = 0; a < ATT_QPW; ++a) {
     const int qi = warp * ATT_QPW + a;
-    if (qi >= nq) break;
-    const float inv = 1.f / l_run[a];
-    bf16* orow = o + static_cast<size_t>(q0 + qi) * dim + h * dh;
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int d = lane + 32 * c;
-      if (d < dh) orow[d] = __float2bfloat16_rn(acc[a][c] * inv);
+    for (int c = 0; c < 4; ++c)
+      if (lane + 32 * c < dh) so[qi * dh + lane + 32 * c] = acc[a][c];
+    if (lane == 0) {
+      sml[2 * qi] = m_run[a];
+      sml[2 * qi + 1] = l_run[a];
     }
   }
+  cluster_sync();
+  const uint32_t so_addr = smem_u32(so), ml_addr = smem_u32(sml);
+  for (int qi = rank + ns * warp; qi < nq; qi += ns * ATT_WARPS) {
+    float ms[8], M = -INFINITY;
+    for (int s = 0; s < ns; ++s) {
+      ms[s] = ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi, s));
+      M = fmaxf(M, ms[s]);
+    }
+    float lsum = 0.f, out[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int s = 0; s < ns; ++s) {
+      const float w = __expf(ms[s] - M);
+      lsum += w * ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi + 4, s));
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        if (lane + 32 * c < dh)
+          out[c] += w * ld_dsmem_f32(mapa_shared(so_addr + 4 * (qi * dh + lane + 32 * c), s));
+    }
+    const float inv = 1.f / lsum;
+    bf16* orow = o + static_cast<size_t>(q0 + qi) * dim + h * dh;
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+      if (lane + 32 * c < dh) orow[lane + 32 * c] = __float2bfloat16_rn(out[c] * inv);
+  }
+  cluster_sync();  // partials stay valid until every CTA of the cluster has read them
 }
 
 }  // namespace
@@ -335,25 +443,21 @@ cudaError_t launch_patchify(const uint8_t* frames, bf16* patches, int sv, int im
   const long long total = static_cast<long long>(sv) * (img_h / patch) * (img_w / patch) * patch;
   const long long blocks = (total + 255) / 256;
   const int grid = static_cast<int>(blocks < 4096 ? blocks : 4096);
-  patchify_kernel<<<grid, 256, 0, s>>>(frames, patches, sv, img_h, img_w, patch, kpad);
-  return cudaGetLastError();
+  return launch_ex(patchify_kernel, dim3(grid), dim3(256), 0, s, 1, frames, patches, sv, img_h, img_w, patch, kpad);
 }
 
 cudaError_t launch_score(const float* e_t, float* e_ref, float* sims, int rows, int dim,
                          int copy_ref, cudaStream_t s) {
   const int grid = min((rows + 7) / 8, 4096);
-  score_kernel<<<grid, 256, 0, s>>>(e_t, e_ref, sims, rows, dim, copy_ref);
-  return cudaGetLastError();
+  return launch_ex(score_kernel, dim3(grid), dim3(256), 0, s, 1, e_t, e_ref, sims, rows, dim, copy_ref);
 }
 
 cudaError_t launch_select(const float* sims, int n_tok, int sv, int mode, float tau, int topk,
                           const ColdMask& cold, int* idx, int* counts, int* cu_rows, int* rowtok,
                           int* done_ctr, int* user_counts, cudaStream_t s) {
   const int threads = (n_tok + 31) / 32 * 32;
-  select_kernel<<<sv, threads, n_tok * sizeof(float), s>>>(sims, n_tok, sv, mode, tau, topk, cold, idx,
-                                                            counts, cu_rows, rowtok, done_ctr,
-                                                            user_counts);
-  return cudaGetLastError();
+  return launch_ex(select_kernel, dim3(sv), dim3(threads), n_tok * sizeof(float), s, 1, sims, n_tok, sv,
+                   mode, tau, topk, cold, idx, counts, cu_rows, rowtok, done_ctr, user_counts);
 }
 
 cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const float* e_t,
@@ -361,32 +465,35 @@ cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const flo
                           int ref_last_refresh, const ColdMask& cold, int max_rows, int grid,
                           cudaStream_t s) {
   grid = max(1, min(grid, (max_rows + 7) / 8));
-  gather_kernel<<<grid, 256, 0, s>>>(cu_rows_total, rowtok, e_t, pos, x, e_ref, n_tok, dim,
-                                     ref_last_refresh, cold);
-  return cudaGetLastError();
+  return launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, 1, cu_rows_total, rowtok, e_t, pos, x,
+                   e_ref, n_tok, dim, ref_last_refresh, cold);
 }
 
 cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma, const float* beta,
                              bf16* y, const int* dst_rowtok, int dim, float eps, int max_rows,
                              int grid, cudaStream_t s) {
   grid = max(1, min(grid, (max_rows + 7) / 8));
-  layernorm_kernel<<<grid, 256, 0, s>>>(rows, x, gamma, beta, y, dst_rowtok, dim, eps);
-  return cudaGetLastError();
+  return launch_ex(layernorm_kernel, dim3(grid), dim3(256), 0, s, 1, rows, x, gamma, beta, y, dst_rowtok,
+                   dim, eps);
+}
+
+cudaError_t attention_setup() {
+  return cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
 }
 
 cudaError_t launch_attention(const bf16* q, const bf16* cache_k, const bf16* cache_v,
                              const int* cu_rows, bf16* o, int sv, int n_tok, int dim, int heads,
                              cudaStream_t s) {
   const int dh = dim / heads;
-  const size_t smem = (2 * ATT_KT * (dh + 1) + ATT_QB * dh) * sizeof(float);
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
-    attr_set = true;
-  }
-  dim3 grid((n_tok + ATT_QB - 1) / ATT_QB, heads, sv);
-  attention_kernel<<<grid, ATT_WARPS * 32, smem, s>>>(q, cache_k, cache_v, cu_rows, o, n_tok, dim, dh);
-  return cudaGetLastError();
+  const size_t smem =
+      (2 * dh * ATT_KT + ATT_QB * dh + ATT_WARPS * ATT_QPW * ATT_KT + 2 * ATT_QB) * sizeof(float);
+  // key splits: about 64 keys each, at most 8 (a portable cluster)
+  int ns = (n_tok + ATT_KT - 1) / ATT_KT;
+  ns = ns < 1 ? 1 : (ns > 8 ? 8 : ns);
+  const int kps = (n_tok + ns - 1) / ns;
+  const dim3 grid(((n_tok + ATT_QB - 1) / ATT_QB) * ns, heads, sv);
+  return launch_ex(attention_kernel, grid, dim3(ATT_WARPS * 32), smem, s, static_cast<unsigned>(ns), q,
+                   cache_k, cache_v, cu_rows, o, n_tok, dim, dh, kps);
 }
 
 }  // namespace ivit

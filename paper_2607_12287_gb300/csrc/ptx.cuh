@@ -18,7 +18,6 @@ enum DeviceError : int {
   kErrWaitTmaFull = 1,    // MMA issuer waited too long for a TMA stage
   kErrWaitSlotEmpty = 2,  // TMA producer waited too long for a free stage
   kErrWaitAccum = 3,      // epilogue waited too long for the accumulator
-  kErrWorkspace = 4,      // split-K workspace too small for the chosen split
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -174,6 +173,49 @@ __device__ __forceinline__ uint32_t idesc_bf16_f32(int m, int n) {
          | (1u << 10)                                 // B format: bf16
          | (static_cast<uint32_t>(n >> 3) << 17)      // N / 8
          | (static_cast<uint32_t>(m >> 4) << 24);     // M / 16
+}
+
+// ------------------------------------------------------------- thread-block clusters
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_nctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+
+// Every thread of every CTA of the cluster arrives and waits; shared-memory writes made
+// before it are visible to the cluster's CTAs after it.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile(
+      "barrier.cluster.arrive.release.aligned;\n\t"
+      "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Address of the same shared-memory variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ float ld_dsmem_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ float4 ld_dsmem_f32x4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
 }
 
 // ------------------------------------------------------ programmatic dependent launch
