@@ -1,0 +1,93 @@
+"""GPU parity at the full workload sizes (the bench's launch configuration), frame by
+frame against the oracle: bit-exact updated-token lists, final tokens within the
+bf16-vs-fp32 tolerance.  Long streams are checked on a prefix; the 448 px batched
+workload compares one stream (two views) with the oracle and every view's list with
+the scene's pixel ground truth."""
+import itertools
+
+import numpy as np
+import pytest
+
+from paper_2607_12287_gb300 import synth
+from tests.gpu_util import assert_tokens_close, run_side_by_side
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def pkg():
+    import paper_2607_12287_gb300 as p
+    p.load()
+    return p
+
+
+def _frames(wl, n):
+    return list(itertools.islice(wl.frames(), n))
+
+
+def test_vit_tiny_square_all_frames(pkg, oracle_mod):
+    wl = synth.WORKLOADS["vit_tiny_224_square"]
+    w = synth.make_weights(wl.shape, 0)
+    frames = _frames(wl, wl.n_frames)
+    stats = run_side_by_side(pkg, oracle_mod, wl.shape, w, frames, check_caches=True)
+    for prev, cur, st in zip(frames, frames[1:], stats[1:]):
+        truth = synth.pixel_changed_patches(prev, cur, wl.shape.patch)
+        assert st[2].tolist() == truth.sum(1).tolist()
+
+
+def test_so400m_1view_prefix(pkg, oracle_mod):
+    wl = synth.WORKLOADS["so400m_224_1view"]
+    w = synth.make_weights(wl.shape, 0)
+    run_side_by_side(pkg, oracle_mod, wl.shape, w, _frames(wl, 4), check_caches=True)
+
+
+def test_so400m_3view_prefix(pkg, oracle_mod):
+    wl = synth.WORKLOADS["so400m_224_3view"]
+    w = synth.make_weights(wl.shape, 0)
+    stats = run_side_by_side(pkg, oracle_mod, wl.shape, w, _frames(wl, 3), 1, 3)
+    assert all(s[2].min() > 0 for s in stats[1:])
+
+
+@pytest.mark.parametrize("fraction", [0.0, 0.05, 0.25, 1.0])
+def test_so400m_sweep_point(pkg, oracle_mod, fraction):
+    wl = synth.sweep_workload(fraction)
+    w = synth.make_weights(wl.shape, 0)
+    frames = _frames(wl, 3)
+    stats = run_side_by_side(pkg, oracle_mod, wl.shape, w, frames, select_mode=wl.select_mode,
+                             topk=wl.topk)
+    for prev, cur, st in zip(frames, frames[1:], stats[1:]):
+        assert st[2].tolist() == [wl.topk]
+        truth = synth.pixel_changed_patches(prev, cur, wl.shape.patch)
+        assert truth.sum() == wl.topk
+
+
+def test_so400m_448_batched(pkg, oracle_mod):
+    import torch
+    wl = synth.WORKLOADS["so400m_448_16x2"]
+    w = synth.make_weights(wl.shape, 0)
+    frames = _frames(wl, 3)
+    enc = pkg.IncrementalViT.for_workload(wl, w)
+    orc = oracle_mod.Oracle(wl.shape, w, 1, 2)  # stream 0 = views 0 and 1
+    try:
+        for t, f in enumerate(frames):
+            fd = torch.from_numpy(f).cuda()
+            if t == 0:
+                out = enc.encode_full(fd)
+                ref = orc.encode_full(f[:2])
+            else:
+                out, counts = enc.encode_incremental(fd)
+                ref, rc, ridx, sims = orc.encode_incremental(f[:2])
+                assert np.abs(sims - wl.threshold).min() > 2e-3
+                counts = counts.cpu().numpy()
+                np.testing.assert_array_equal(counts[:2], rc)
+                for v in range(2):
+                    np.testing.assert_array_equal(enc.changed(v).cpu().numpy(), ridx[v, :rc[v]])
+                truth = synth.pixel_changed_patches(frames[t - 1], f, wl.shape.patch)
+                for v in range(wl.sv):
+                    np.testing.assert_array_equal(enc.changed(v).cpu().numpy(), np.nonzero(truth[v])[0],
+                                                  err_msg=f"view {v}")
+            assert_tokens_close(out[:2].float().cpu().numpy(), ref, f"frame {t}")
+        assert enc.device_status() == 0
+    finally:
+        enc.close()
+        orc.close()
