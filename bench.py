@@ -138,6 +138,23 @@ def make_frames(wl, n: int):
     return [np.ascontiguousarray(f) for f in wl.frames(n)]
 
 
+def replica_workload(wl, rank: int):
+    """Weak scaling: every rank encodes its own camera streams (the same scene recipe
+    with its own seed); ranks exchange nothing on the data path."""
+    import dataclasses
+    return dataclasses.replace(wl, seed=wl.seed + 1000 * rank) if rank else wl
+
+
+def max_over_ranks(value: float, dist, device=None) -> float:
+    """The slowest rank's time (the job finishes when every replica has)."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def cpu_baseline(wl, weights, frames, budget_s: float = 20.0) -> dict:
     """The oracle as it stands, on this host's cores: an untimed full encode of frame 0,
     then incremental frames timed until ``budget_s`` is spent (at least one)."""
@@ -223,6 +240,7 @@ def main() -> None:
 
     import paper_2607_12287_gb300 as pkg
     dev = torch.device("cuda", local_rank)
+    wl = replica_workload(wl, rank)
     weights = synth.make_weights(wl.shape, 0)
     n_frames = 1 + args.warmup + args.steps
     frames = make_frames(wl, n_frames)
@@ -252,11 +270,7 @@ def main() -> None:
         e1.synchronize()
         ms = e0.elapsed_time(e1)
         barrier()
-        if dist is not None:
-            m = torch.tensor([ms], device=dev)
-            dist.all_reduce(m, op=dist.ReduceOp.MAX)
-            ms = float(m.item())
-        return ms
+        return max_over_ranks(ms, dist, dev)
 
     def inc_step(t):
         pkg.ivit_encode_incremental(enc.h, frames_dev[t], out, counts[t], stream)
