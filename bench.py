@@ -256,6 +256,8 @@ def main() -> None:
             dist.barrier()
         torch.cuda.synchronize(dev)
 
+    host_ms = {}
+
     def timed(fn_step, label):
         """Full encode of frame 0, warm-up frames, then K timed steps (CUDA events)."""
         enc.encode_full(frames_dev[0], out)
@@ -264,8 +266,10 @@ def main() -> None:
         barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
+        h0 = time.perf_counter()
         for t in range(args.steps):
             fn_step(1 + args.warmup + t)
+        host_ms[label] = 1e3 * (time.perf_counter() - h0) / args.steps
         e1.record(stream)
         e1.synchronize()
         ms = e0.elapsed_time(e1)
@@ -340,6 +344,7 @@ def main() -> None:
                      "traffic": traffic, "peak_source": peaks["source"],
                      "launches_timed": gemm_n, "avg_launch_us": 1e3 * gemm_ms / gemm_n if gemm_n else None,
                      "algorithmic_bytes_per_launch": gemm_bytes / gemm_n if gemm_n else None},
+        "host_enqueue_ms_per_step": host_ms,
         "gpu_launches": int(launches_per_step * args.steps),
         "launches_per_step": int(launches_per_step),
         "device_status": status,

@@ -49,7 +49,7 @@ extern "C" {
 
 /* Encoder + selection configuration.
  * Supported by the kernels: patch >= 1 dividing img_h and img_w; N <= 1024;
- * dim % 64 == 0 and heads dividing dim with head_dim = dim/heads a multiple of 8,
+ * dim % 64 == 0, dim <= 2048, heads dividing dim with head_dim = dim/heads a multiple of 8,
  * at most 128; mlp_dim % 8 == 0; SV <= 4096. */
 typedef struct ivit_config {
   int32_t img_h, img_w;  /* frame size in pixels */

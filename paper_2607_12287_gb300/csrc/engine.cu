@@ -163,7 +163,7 @@ const char* validate(const ivit_config* c) {
   if (c->img_h % c->patch || c->img_w % c->patch) return "patch must divide img_h and img_w";
   const long long n = static_cast<long long>(c->img_h / c->patch) * (c->img_w / c->patch);
   if (n > 1024) return "at most 1024 tokens per view";
-  if (c->dim <= 0 || c->dim % 64) return "dim must be a positive multiple of 64";
+  if (c->dim <= 0 || c->dim % 64 || c->dim > 2048) return "dim must be a multiple of 64 in [64, 2048]";
   if (c->heads <= 0 || c->dim % c->heads) return "heads must divide dim";
   const int dh = c->dim / c->heads;
   if (dh % 8 || dh > 128) return "head_dim must be a multiple of 8 and at most 128";
@@ -490,7 +490,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
       a.epi.dim = D;
       if (int r = gemm(h, plan[kGemmQKV], w.tm_qkv, h->tm_xn, a, s)) return r;
     }
-    IVIT_CK(h, ivit::launch_attention(h->q, ck, cv, h->cu_rows, h->o, SV, N, D, h->H, s));
+    IVIT_CK(h, ivit::launch_attention(h->q, ck, cv, h->cu_rows, h->rowtok, h->o, SV, N, D, h->H, s));
     ++h->launches;
     {
       ivit::GemmArgs a;

@@ -118,8 +118,10 @@ cudaError_t attention_setup();
 
 // O[r] = softmax(Q[r] K_v^T / sqrt(dh)) V_v per head, for the packed query rows r of
 // each view v (cu_rows), over the N cached keys/values of that view.
+// rowtok lists the updated tokens (packed row -> v*N + i): their keys are re-read after
+// the wait on the QKV kernel, every other key may be read before it.
 cudaError_t launch_attention(const bf16* q, const bf16* cache_k, const bf16* cache_v,
-                             const int* cu_rows, bf16* o, int sv, int n_tok, int dim, int heads,
-                             cudaStream_t s);
+                             const int* cu_rows, const int* rowtok, bf16* o, int sv, int n_tok,
+                             int dim, int heads, cudaStream_t s);
 
 }  // namespace ivit

@@ -203,14 +203,23 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, const float* __r
                                  const float* __restrict__ gamma, const float* __restrict__ beta,
                                  bf16* __restrict__ y, const int* __restrict__ dst_rowtok, int dim,
                                  float eps) {
-  pdl_wait();
-  pdl_launch_dependents();
-  const int rows = *nrows;
   const int warps = blockDim.x >> 5;
   const int lane = threadIdx.x & 31;
   const int n4 = dim / 4;
+  // Before waiting on the previous kernel: the affine parameters (constant) and the row
+  // count (written by the selection kernel, at least two launches back).
   const float4* g4 = reinterpret_cast<const float4*>(gamma);
   const float4* b4 = reinterpret_cast<const float4*>(beta);
+  float4 g[LN_MAX_F4_PER_LANE], bb[LN_MAX_F4_PER_LANE];
+#pragma unroll
+  for (int i = 0; i < LN_MAX_F4_PER_LANE; ++i) {
+    const int c = lane + 32 * i;
+    g[i] = c < n4 ? g4[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+    bb[i] = c < n4 ? b4[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  const int rows = *nrows;
+  pdl_wait();
+  pdl_launch_dependents();
   for (int r = blockIdx.x * warps + (threadIdx.x >> 5); r < rows; r += gridDim.x * warps) {
     const float4* xr = reinterpret_cast<const float4*>(x + static_cast<size_t>(r) * dim);
     float4 v[LN_MAX_F4_PER_LANE];
@@ -237,9 +246,11 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, const float* __r
     for (int i = 0; i < LN_MAX_F4_PER_LANE; ++i) {
       const int c = lane + 32 * i;
       if (c < n4) {
-        const float4 g = g4[c], b = b4[c], u = v[i];
-        yr[2 * c] = __floats2bfloat162_rn(g.x * (u.x - mean) * rstd + b.x, g.y * (u.y - mean) * rstd + b.y);
-        yr[2 * c + 1] = __floats2bfloat162_rn(g.z * (u.z - mean) * rstd + b.z, g.w * (u.w - mean) * rstd + b.w);
+        const float4 u = v[i];
+        yr[2 * c] = __floats2bfloat162_rn(g[i].x * (u.x - mean) * rstd + bb[i].x,
+                                          g[i].y * (u.y - mean) * rstd + bb[i].y);
+        yr[2 * c + 1] = __floats2bfloat162_rn(g[i].z * (u.z - mean) * rstd + bb[i].z,
+                                              g[i].w * (u.w - mean) * rstd + bb[i].w);
       }
     }
   }
@@ -250,45 +261,86 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, const float* __r
 // K/V with this call's updated rows already written), per head:
 //   O = softmax(Q K^T / sqrt(dh)) V.
 // Grid: (query block x key split, head, view); the key splits of one query block form
-// a thread-block cluster.  Each CTA streams its key range in tiles of ATT_KT through
-// shared memory (16-byte loads; K stored transposed so lanes read consecutive keys),
-// keeps an online softmax per query (running max m, sum l, output row in registers),
-// then the cluster merges its partial (m, l, o) through distributed shared memory:
-//   M = max_s m_s,  O = sum_s exp(m_s - M) o_s / sum_s exp(m_s - M) l_s.
-// Warp w owns queries 4w..4w+3 of the block; lane owns keys lane, lane+32 of a tile
-// for the scores and output dims lane + 32c for P V.
+// a thread-block cluster.  Each CTA keeps its whole key range (at most ATT_KR keys) in
+// shared memory as bf16, K transposed so lanes read consecutive keys.  The range is
+// loaded before waiting on the QKV kernel (the cached keys of reused tokens do not
+// change), and only the keys of this call's updated tokens are read again after it.
+// Per query: online softmax over 64-key sub-tiles (running max m, sum l, output row in
+// registers), then the cluster merges its partial (m, l, o) through distributed
+// shared memory:  M = max_s m_s,  O = sum_s exp(m_s - M) o_s / sum_s exp(m_s - M) l_s.
+// Warp w owns queries 4w..4w+3; lane owns keys lane, lane+32 of a sub-tile for the
+// scores and output dims lane + 32c for P V.
 constexpr int ATT_WARPS = 8;
 constexpr int ATT_QPW = 4;
 constexpr int ATT_QB = ATT_WARPS * ATT_QPW;
-constexpr int ATT_KT = 64;
+constexpr int ATT_KT = 64;    // keys per softmax sub-tile
+constexpr int ATT_KR = 128;   // max keys per CTA (key split)
+
+__device__ __forceinline__ void att_store_key(bf16* skT, bf16* sv, int dh, int j, int c, uint4 uk,
+                                              uint4 uv) {
+  const bf16* k8 = reinterpret_cast<const bf16*>(&uk);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) skT[(c * 8 + i) * ATT_KR + j] = k8[i];
+  *reinterpret_cast<uint4*>(sv + j * dh + c * 8) = uv;
+}
 
 __global__ void __launch_bounds__(ATT_WARPS * 32)
     attention_kernel(const bf16* __restrict__ q, const bf16* __restrict__ cache_k,
                      const bf16* __restrict__ cache_v, const int* __restrict__ cu_rows,
-                     bf16* __restrict__ o, int N, int dim, int dh, int keys_per_split) {
-  pdl_wait();
-  pdl_launch_dependents();
+                     const int* __restrict__ rowtok, bf16* __restrict__ o, int N, int dim, int dh,
+                     int keys_per_split) {
   extern __shared__ float sm[];
-  float* skT = sm;                          // [dh][KT]   (after the key loop: partial o [QB][dh])
-  float* sv = skT + dh * ATT_KT;            // [KT][dh]
-  float* sq = sv + ATT_KT * dh;             // [QB][dh]
-  float* sp = sq + ATT_QB * dh;             // [WARPS][QPW][KT]
-  float* sml = sp + ATT_WARPS * ATT_QPW * ATT_KT;  // [QB][2]
+  float* sq = sm;                                   // [QB][dh] fp32, pre-scaled
+  float* sp = sq + ATT_QB * dh;                     // [WARPS][QPW][KT]
+  float* sml = sp + ATT_WARPS * ATT_QPW * ATT_KT;   // [QB][2]
+  float* so = sml + 2 * ATT_QB;                     // [QB][dh] partial outputs
+  bf16* skT = reinterpret_cast<bf16*>(so + ATT_QB * dh);  // [dh][KR]
+  bf16* sv = skT + dh * ATT_KR;                           // [KR][dh]
   const int ns = static_cast<int>(cluster_nctarank());
   const int rank = static_cast<int>(cluster_ctarank());
   const int v = blockIdx.z, h = blockIdx.y, qb = blockIdx.x / ns;
-  const int r_begin = cu_rows[v], r_end = cu_rows[v + 1];
-  const int q0 = r_begin + qb * ATT_QB;
-  if (q0 >= r_end) return;  // the whole cluster shares qb, so it leaves together
-  const int nq = min(ATT_QB, r_end - q0);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int dh8 = dh / 8;
-  const float scale = rsqrtf(static_cast<float>(dh));
+  // Row ranges come from the selection kernel (complete before this grid can start).
+  const int r_begin = cu_rows[v], r_end = cu_rows[v + 1];
+  const int q0 = r_begin + qb * ATT_QB;
+  if (q0 >= r_end) {  // the whole cluster shares qb, so it leaves together
+    pdl_wait();
+    pdl_launch_dependents();
+    return;
+  }
+  const int nq = min(ATT_QB, r_end - q0);
   const int k_begin = rank * keys_per_split, k_end = min(N, k_begin + keys_per_split);
+  const int nkr = k_end - k_begin;
+  const size_t vbase = static_cast<size_t>(v) * N;
 
+  // cached keys/values of the range (reused tokens' rows are final already)
+  for (int e = tid; e < ATT_KR * dh8; e += blockDim.x) {
+    const int j = e % ATT_KR, c = e / ATT_KR;
+    if (j < nkr) {
+      const size_t g = (vbase + k_begin + j) * dim + h * dh + c * 8;
+      att_store_key(skT, sv, dh, j, c, *reinterpret_cast<const uint4*>(cache_k + g),
+                    *reinterpret_cast<const uint4*>(cache_v + g));
+    }
+  }
+  pdl_wait();  // the QKV kernel's queries and new K/V rows are visible from here
+  pdl_launch_dependents();
+
+  // re-read the keys this call updated (tokens of view v listed in rowtok)
+  const int n_upd = r_end - r_begin;
+  for (int e = tid; e < n_upd * dh8; e += blockDim.x) {
+    const int r = e / dh8, c = e % dh8;
+    const int j = rowtok[r_begin + r] - static_cast<int>(vbase) - k_begin;
+    if (j >= 0 && j < nkr) {
+      const size_t g = (vbase + k_begin + j) * dim + h * dh + c * 8;
+      att_store_key(skT, sv, dh, j, c, __ldcg(reinterpret_cast<const uint4*>(cache_k + g)),
+                    __ldcg(reinterpret_cast<const uint4*>(cache_v + g)));
+    }
+  }
+  const float scale = rsqrtf(static_cast<float>(dh));
   for (int e = tid; e < nq * dh8; e += blockDim.x) {
     const int qi = e / dh8, c = e % dh8;
-    const uint4 u = *reinterpret_cast<const uint4*>(q + static_cast<size_t>(q0 + qi) * dim + h * dh + c * 8);
+    const uint4 u = __ldcg(reinterpret_cast<const uint4*>(q + static_cast<size_t>(q0 + qi) * dim + h * dh + c * 8));
     const __nv_bfloat162* b2 = reinterpret_cast<const __nv_bfloat162*>(&u);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -297,6 +349,7 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
       sq[qi * dh + c * 8 + 2 * i + 1] = f.y * scale;
     }
   }
+  __syncthreads();
 
   float m_run[ATT_QPW], l_run[ATT_QPW], acc[ATT_QPW][4];
 #pragma unroll
@@ -306,44 +359,18 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc[a][c] = 0.f;
   }
-  const size_t vbase = static_cast<size_t>(v) * N;
   float* spw = sp + warp * ATT_QPW * ATT_KT;
+  const float* qw = sq + warp * ATT_QPW * dh;
+  const bool warp_active = warp * ATT_QPW < nq;
 
-  for (int k0 = k_begin; k0 < k_end; k0 += ATT_KT) {
-    const int nk = min(ATT_KT, k_end - k0);
-    __syncthreads();
-    for (int e = tid; e < ATT_KT * dh8; e += blockDim.x) {
-      const int j = e % ATT_KT, c = e / ATT_KT;
-      if (j < nk) {
-        const size_t g = (vbase + k0 + j) * dim + h * dh + c * 8;
-        const uint4 uk = *reinterpret_cast<const uint4*>(cache_k + g);
-        const uint4 uv = *reinterpret_cast<const uint4*>(cache_v + g);
-        const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&uk);
-        const __nv_bfloat162* v2 = reinterpret_cast<const __nv_bfloat162*>(&uv);
-        float4* vd = reinterpret_cast<float4*>(sv + j * dh + c * 8);
-        float tv[8];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float2 fk = __bfloat1622float2(k2[i]);
-          skT[(c * 8 + 2 * i) * ATT_KT + j] = fk.x;
-          skT[(c * 8 + 2 * i + 1) * ATT_KT + j] = fk.y;
-          const float2 fv = __bfloat1622float2(v2[i]);
-          tv[2 * i] = fv.x;
-          tv[2 * i + 1] = fv.y;
-        }
-        vd[0] = make_float4(tv[0], tv[1], tv[2], tv[3]);
-        vd[1] = make_float4(tv[4], tv[5], tv[6], tv[7]);
-      }
-    }
-    __syncthreads();
-
-    // scores of this warp's queries against the tile (lane: keys lane and lane + 32)
+  for (int t0 = 0; t0 < nkr && warp_active; t0 += ATT_KT) {
+    const int nk = min(ATT_KT, nkr - t0);
     float s0[ATT_QPW], s1[ATT_QPW];
 #pragma unroll
     for (int a = 0; a < ATT_QPW; ++a) s0[a] = s1[a] = 0.f;
-    const float* qw = sq + warp * ATT_QPW * dh;
     for (int d = 0; d < dh; ++d) {
-      const float k0v = skT[d * ATT_KT + lane], k1v = skT[d * ATT_KT + lane + 32];
+      const float k0v = __bfloat162float(skT[d * ATT_KR + t0 + lane]);
+      const float k1v = __bfloat162float(skT[d * ATT_KR + t0 + lane + 32]);
 #pragma unroll
       for (int a = 0; a < ATT_QPW; ++a) {
         const float qv = qw[a * dh + d];
@@ -370,7 +397,8 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
     for (int j = 0; j < nk; ++j) {
       float vv[4];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) vv[c] = (lane + 32 * c < dh) ? sv[j * dh + lane + 32 * c] : 0.f;
+      for (int c = 0; c < 4; ++c)
+        vv[c] = (lane + 32 * c < dh) ? __bfloat162float(sv[(t0 + j) * dh + lane + 32 * c]) : 0.f;
 #pragma unroll
       for (int a = 0; a < ATT_QPW; ++a) {
         const float pj = spw[a * ATT_KT + j];
@@ -397,8 +425,6 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
   }
 
   // partial (m, l, o) of every query of the block, then a cluster-wide merge
-  __syncthreads();
-  float* so = skT;  // [QB][dh]
 #pragma unroll
   for (int a = 0; a < ATT_QPW; ++a) {
     const int qi = warp * ATT_QPW + a;
@@ -413,14 +439,11 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
   cluster_sync();
   const uint32_t so_addr = smem_u32(so), ml_addr = smem_u32(sml);
   for (int qi = rank + ns * warp; qi < nq; qi += ns * ATT_WARPS) {
-    float ms[8], M = -INFINITY;
-    for (int s = 0; s < ns; ++s) {
-      ms[s] = ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi, s));
-      M = fmaxf(M, ms[s]);
-    }
+    float M = -INFINITY;
+    for (int s = 0; s < ns; ++s) M = fmaxf(M, ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi, s)));
     float lsum = 0.f, out[4] = {0.f, 0.f, 0.f, 0.f};
     for (int s = 0; s < ns; ++s) {
-      const float w = __expf(ms[s] - M);
+      const float w = __expf(ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi, s)) - M);
       lsum += w * ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi + 4, s));
 #pragma unroll
       for (int c = 0; c < 4; ++c)
@@ -477,23 +500,27 @@ cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma
                    dim, eps);
 }
 
+size_t attention_smem(int dh) {
+  return (2 * ATT_QB * dh + ATT_WARPS * ATT_QPW * ATT_KT + 2 * ATT_QB) * sizeof(float) +
+         2 * static_cast<size_t>(dh) * ATT_KR * sizeof(bf16);
+}
+
 cudaError_t attention_setup() {
-  return cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
+  return cudaFuncSetAttribute(attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(attention_smem(128)));
 }
 
 cudaError_t launch_attention(const bf16* q, const bf16* cache_k, const bf16* cache_v,
-                             const int* cu_rows, bf16* o, int sv, int n_tok, int dim, int heads,
-                             cudaStream_t s) {
+                             const int* cu_rows, const int* rowtok, bf16* o, int sv, int n_tok,
+                             int dim, int heads, cudaStream_t s) {
   const int dh = dim / heads;
-  const size_t smem =
-      (2 * dh * ATT_KT + ATT_QB * dh + ATT_WARPS * ATT_QPW * ATT_KT + 2 * ATT_QB) * sizeof(float);
-  // key splits: about 64 keys each, at most 8 (a portable cluster)
+  // key splits of about 64 keys (at most 128, at most 8 CTAs: a portable cluster)
   int ns = (n_tok + ATT_KT - 1) / ATT_KT;
   ns = ns < 1 ? 1 : (ns > 8 ? 8 : ns);
   const int kps = (n_tok + ns - 1) / ns;
   const dim3 grid(((n_tok + ATT_QB - 1) / ATT_QB) * ns, heads, sv);
-  return launch_ex(attention_kernel, grid, dim3(ATT_WARPS * 32), smem, s, static_cast<unsigned>(ns), q,
-                   cache_k, cache_v, cu_rows, o, n_tok, dim, dh, kps);
+  return launch_ex(attention_kernel, grid, dim3(ATT_WARPS * 32), attention_smem(dh), s,
+                   static_cast<unsigned>(ns), q, cache_k, cache_v, cu_rows, rowtok, o, n_tok, dim, dh, kps);
 }
 
 }  // namespace ivit
