@@ -131,6 +131,12 @@ int ivit_profile_read(ivit_handle* h, double* gemm_ms_total, int64_t* gemm_launc
  * wait expired, the kernel skipped its work and returned).  Synchronises `stream`. */
 int ivit_device_status(ivit_handle* h, void* stream);
 
+/* Execution paths (chosen at create; the environment variable IVIT_PATH=kernels or
+ * IVIT_PATH=persistent overrides the default): one kernel per operation, chained with
+ * programmatic dependent launch and replayed as a CUDA graph (default for dim > 384),
+ * or every transformer block of a call in one persistent cooperative kernel with grid
+ * barriers (default for dim <= 384, where per-operation launches dominate). */
+
 /* Number of the library's kernel launches made by the last encode call. */
 int64_t ivit_last_launch_count(const ivit_handle* h);
 

@@ -55,9 +55,9 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 }
 
 // bf16 2-D tensor [rows][inner] with the given row stride; box = box_inner x box_rows,
-// 128-byte swizzle (box_inner * 2 == 128), out-of-bounds elements read as zero.
+// 128-byte swizzle (box_inner * 2 == 128) or dense rows, out-of-bounds elements read as 0.
 bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint64_t stride_bytes,
-              uint32_t box_inner, uint32_t box_rows) {
+              uint32_t box_inner, uint32_t box_rows, bool swizzle = true) {
   auto enc = tensor_map_encoder();
   if (!enc) return false;
   cuuint64_t dims[2] = {inner, rows};
@@ -65,7 +65,7 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, u
   cuuint32_t box[2] = {box_inner, box_rows};
   cuuint32_t estr[2] = {1, 1};
   return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -120,6 +120,13 @@ struct ivit_handle {
 
   std::vector<uint8_t> cold;
   int64_t launches = 0;
+
+  // Persistent encoder (all blocks in one cooperative launch) for small row tiles.
+  bool persistent = false;
+  size_t pt_smem = 0;
+  int pt_grid = 0;
+  void* pt_mem = nullptr;  // device: tensor maps, layer parameters, partials, barrier words
+  ivit::PersistentArgs pt_args{};
 
   // CUDA graphs of the full and the steady-state incremental chain.  Inputs and outputs
   // are staged through handle-owned buffers (copies outside the graph), so the graph's
@@ -210,6 +217,97 @@ GemmPlan plan_gemm(int num_sms, int bn, int n_out, int k, int m_expected) {
     }
   }
   return best;
+}
+
+// Prepares the persistent encoder when its shared memory fits (attention keeps a whole
+// view's keys and values of one head resident, so N * head_dim is bounded).
+int setup_persistent(ivit_handle* h) {
+  // IVIT_PATH=kernels / IVIT_PATH=persistent override the choice made from the shape.
+  // Default: small encoders (dim <= 384), whose per-layer kernels are launch-bound.
+  const char* path = std::getenv("IVIT_PATH");
+  if (path && std::strcmp(path, "kernels") == 0) return IVIT_OK;
+  if (!(path && std::strcmp(path, "persistent") == 0) && h->D > 384) return IVIT_OK;
+  const int dh = h->D / h->H;
+  const size_t smem = ivit::persistent_smem_bytes(h->N, dh);
+  if (smem > 227 * 1024 || h->D > 2048 || h->N > 256) return IVIT_OK;
+  IVIT_CK(h, ivit::persistent_setup(smem));
+  const int grid = std::min(h->num_sms, ivit::persistent_max_ctas(smem));
+  if (grid < 1) return IVIT_OK;
+  const int L = h->L;
+  // partial slots: at most one item per CTA with K split, else one per tile
+  const int n_tt = (h->M_max + 63) / 64;
+  const int max_tiles = std::max({(3 * h->D + 127) / 128, (h->F + 127) / 128}) * n_tt;
+  const int max_items = std::max(grid, max_tiles);
+  Arena pa;
+  const size_t o_w = pa.take(sizeof(CUtensorMap) * 4 * L), o_x = pa.take(sizeof(CUtensorMap) * 3);
+  const size_t o_kv = pa.take(sizeof(CUtensorMap) * 2 * L);
+  const size_t o_lp = pa.take(sizeof(ivit::LayerParams) * L);
+  const size_t o_part = pa.take(ivit::persistent_part_floats(max_items) * sizeof(float));
+  const size_t o_bar = pa.take(4 * sizeof(unsigned));
+  IVIT_CK(h, cudaMalloc(&h->pt_mem, pa.size));
+  IVIT_CK(h, cudaMemset(h->pt_mem, 0, pa.size));
+  pa.base = static_cast<char*>(h->pt_mem);
+  std::vector<CUtensorMap> wm(4 * L);
+  std::vector<ivit::LayerParams> lp(L);
+  for (int l = 0; l < L; ++l) {
+    const LayerW& w = h->layers[l];
+    wm[4 * l + 0] = w.tm_qkv;
+    wm[4 * l + 1] = w.tm_o;
+    wm[4 * l + 2] = w.tm_1;
+    wm[4 * l + 3] = w.tm_2;
+    lp[l] = ivit::LayerParams{w.bqkv, w.bo, w.b1, w.b2, w.ln1g, w.ln1b, w.ln2g, w.ln2b};
+  }
+  const CUtensorMap xm[3] = {h->tm_xn, h->tm_o, h->tm_h};
+  std::vector<CUtensorMap> kvm(2 * L);
+  for (int l = 0; l < L; ++l) {
+    const size_t off = static_cast<size_t>(l) * h->M_max * h->D;
+    if (!make_map(&kvm[2 * l], h->cacheK + off, h->D, h->M_max, h->D * 2, dh, h->N, false) ||
+        !make_map(&kvm[2 * l + 1], h->cacheV + off, h->D, h->M_max, h->D * 2, dh, h->N, false))
+      return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for a cache tile");
+  }
+  IVIT_CK(h, cudaMemcpy(pa.base + o_kv, kvm.data(), sizeof(CUtensorMap) * 2 * L, cudaMemcpyHostToDevice));
+  IVIT_CK(h, cudaMemcpy(pa.base + o_w, wm.data(), sizeof(CUtensorMap) * 4 * L, cudaMemcpyHostToDevice));
+  IVIT_CK(h, cudaMemcpy(pa.base + o_x, xm, sizeof(xm), cudaMemcpyHostToDevice));
+  IVIT_CK(h, cudaMemcpy(pa.base + o_lp, lp.data(), sizeof(ivit::LayerParams) * L, cudaMemcpyHostToDevice));
+  ivit::PersistentArgs& a = h->pt_args;
+  a.N = h->N;
+  a.D = h->D;
+  a.F = h->F;
+  a.H = h->H;
+  a.dh = dh;
+  a.L = L;
+  a.SV = h->SV;
+  a.M_max = h->M_max;
+  a.eps = h->cfg.ln_eps;
+  a.gelu = h->cfg.gelu;
+  a.cu_rows = h->cu_rows;
+  a.rowtok = h->rowtok;
+  a.wmaps = pa.at<CUtensorMap>(o_w);
+  a.xmaps = pa.at<CUtensorMap>(o_x);
+  a.kvmaps = pa.at<CUtensorMap>(o_kv);
+  a.layers = pa.at<ivit::LayerParams>(o_lp);
+  a.lnfg = h->lnfg;
+  a.lnfb = h->lnfb;
+  a.x = h->x;
+  a.xn = h->xn;
+  a.q = h->q;
+  a.o = h->o;
+  a.h = h->hbuf;
+  a.cacheK = h->cacheK;
+  a.cacheV = h->cacheV;
+  a.tok_out = h->tok_out;
+  a.part = pa.at<float>(o_part);
+  a.gbar = pa.at<unsigned>(o_bar);
+  a.err = h->err;
+  a.trace = nullptr;
+  if (std::getenv("IVIT_TRACE")) {
+    IVIT_CK(h, cudaMalloc(&a.trace, 4096 * sizeof(unsigned long long)));
+    IVIT_CK(h, cudaMemset(a.trace, 0, 4096 * sizeof(unsigned long long)));
+  }
+  h->pt_smem = smem;
+  h->pt_grid = grid;
+  h->persistent = true;
+  return IVIT_OK;
 }
 
 int setup(ivit_handle* h, const uint16_t* wb) {
@@ -378,11 +476,16 @@ int setup(ivit_handle* h, const uint16_t* wb) {
       !make_map(&h->tm_o, h->o, D, M, D * 2, 64, 32) ||
       !make_map(&h->tm_h, h->hbuf, F, M, F * 2, 64, 32))
     return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
+  if (int r = setup_persistent(h)) return r;
   IVIT_CK(h, cudaDeviceSynchronize());
   return IVIT_OK;
 }
 
 void release(ivit_handle* h) {
+  if (h->pt_args.trace) cudaFree(h->pt_args.trace);
+  h->pt_args.trace = nullptr;
+  if (h->pt_mem) cudaFree(h->pt_mem);
+  h->pt_mem = nullptr;
   if (h->graph_full) cudaGraphExecDestroy(h->graph_full);
   if (h->graph_inc) cudaGraphExecDestroy(h->graph_inc);
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
@@ -430,6 +533,27 @@ int gemm(ivit_handle* h, const GemmPlan& plan, const CUtensorMap& tw, const CUte
   return IVIT_OK;
 }
 
+// Debug aid (IVIT_TRACE): mean time of each phase kind of the last persistent launch.
+void print_trace(ivit_handle* h, cudaStream_t s) {
+  std::vector<unsigned long long> t(4096);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return;
+  cudaMemcpy(t.data(), h->pt_args.trace, t.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost);
+  const int n = static_cast<int>(t[0]);
+  static const char* names[9] = {"qkv gemm", "qkv reduce", "attention", "out gemm", "out red+LN2",
+                                 "up gemm", "up reduce", "down gemm", "down red+LN"};
+  double acc[9] = {0};
+  int cnt[9] = {0};
+  for (int i = 2; i < n; ++i) {  // entry 1 = start, entry 2 = after the first LN phase
+    const int k = (i - 2) % 9;
+    acc[k] += 1e-3 * static_cast<double>(t[1 + i] - t[i]);
+    ++cnt[k];
+  }
+  std::fprintf(stderr, "ivit trace: %d phases, total %.1f us, first LN %.1f us\n", n - 1,
+               1e-3 * static_cast<double>(t[n] - t[1]), 1e-3 * static_cast<double>(t[2] - t[1]));
+  for (int k = 0; k < 9; ++k)
+    if (cnt[k]) std::fprintf(stderr, "  %-12s %6.2f us x %d\n", names[k], acc[k] / cnt[k], cnt[k]);
+}
+
 // Enqueues the whole chain for one frame per view on `s` (eagerly or under capture).
 int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool full, cudaStream_t s) {
   const ivit_config& c = h->cfg;
@@ -468,6 +592,17 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
                                  c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
   ++h->launches;
 
+  if (h->persistent) {
+    IVIT_CK(h, cudaMemsetAsync(h->pt_args.gbar, 0, 4 * sizeof(unsigned), s));
+    IVIT_CK(h, ivit::launch_persistent(h->pt_args, h->pt_grid, h->pt_smem, s));
+    ++h->launches;
+    if (h->pt_args.trace && !h->profiling) {
+      cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+      cudaStreamIsCapturing(s, &cs);
+      if (cs == cudaStreamCaptureStatusNone) print_trace(h, s);
+    }
+    return IVIT_OK;
+  }
   for (int l = 0; l < h->L; ++l) {
     const LayerW& w = h->layers[l];
     bf16* ck = h->cacheK + static_cast<size_t>(l) * M * D;

@@ -87,6 +87,37 @@ int gemm_max_clusters(int bn_max, int csize);
 cudaError_t launch_gemm(int bn_max, const CUtensorMap& tm_w, const CUtensorMap& tm_x,
                         const GemmArgs& a, int n_clusters, int csize, cudaStream_t s);
 
+// ------------------------------------------------------- persistent encoder (small M)
+struct LayerParams {
+  const float *bqkv, *bo, *b1, *b2, *ln1g, *ln1b, *ln2g, *ln2b;
+};
+
+struct PersistentArgs {
+  int N, D, F, H, dh, L, SV, M_max;
+  float eps;
+  int gelu;
+  const int* cu_rows;             // [SV+1], cu_rows[SV] = updated rows M
+  const int* rowtok;              // [M] packed row -> token v*N + i
+  const CUtensorMap* wmaps;       // [L][4] weight maps (qkv, out, up, down), device memory
+  const CUtensorMap* xmaps;       // [3] activation maps (xn, o, h), device memory
+  const CUtensorMap* kvmaps;      // [L][2] key/value cache maps, box [N rows][dh], device memory
+  const LayerParams* layers;      // [L], device memory
+  const float *lnfg, *lnfb;
+  float* x;                       // fp32 residual stream [M_max][D]
+  bf16 *xn, *q, *o, *h, *cacheK, *cacheV, *tok_out;
+  float* part;                    // K-split partial tiles
+  unsigned* gbar;                 // [count, generation, abort], zero at launch
+  int* err;
+  unsigned long long* trace;      // optional: [0] count, then phase-exit times of CTA 0
+};
+
+size_t persistent_smem_bytes(int n_tok, int head_dim);
+size_t persistent_part_floats(int max_items);
+cudaError_t persistent_setup(size_t smem);
+int persistent_max_ctas(size_t smem);
+// Cooperative launch (all CTAs resident); fails if the grid cannot be resident.
+cudaError_t launch_persistent(const PersistentArgs& a, int grid, size_t smem, cudaStream_t s);
+
 // ------------------------------------------------------------------- other kernels
 struct ColdMask {
   uint32_t bits[128];  // bit v set: view v is cold (updates every token); up to 4096 views

@@ -18,6 +18,7 @@ enum DeviceError : int {
   kErrWaitTmaFull = 1,    // MMA issuer waited too long for a TMA stage
   kErrWaitSlotEmpty = 2,  // TMA producer waited too long for a free stage
   kErrWaitAccum = 3,      // epilogue waited too long for the accumulator
+  kErrGridBarrier = 4,    // a persistent kernel's grid barrier did not complete in time
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -216,6 +217,30 @@ __device__ __forceinline__ float4 ld_dsmem_f32x4(uint32_t addr) {
                : "r"(addr)
                : "memory");
   return v;
+}
+
+// ------------------------------------------------------------- global-memory sync
+__device__ __forceinline__ unsigned ld_acquire_u32(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ unsigned atom_add_acq_rel_u32(unsigned* p, unsigned v) {
+  unsigned r;
+  asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], %2;" : "=r"(r) : "l"(p), "r"(v) : "memory");
+  return r;
+}
+
+// Second arrival on a two-arrival stage barrier without adding transaction bytes.
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// Orders this thread's earlier generic-proxy view of global memory before its later
+// async-proxy (TMA) accesses.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
 // ------------------------------------------------------ programmatic dependent launch

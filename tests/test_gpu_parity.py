@@ -125,3 +125,20 @@ def test_last_refresh_reference(pkg, oracle_mod):
     frames = list(synth.stream_random(shape, 2, 4, 20, change_p=0.3))
     run_side_by_side(pkg, oracle_mod, shape, w, frames, 1, 2,
                      ref_mode=synth.REF_LAST_REFRESH, check_caches=True)
+
+
+@pytest.fixture
+def forced_path(request, monkeypatch):
+    monkeypatch.setenv("IVIT_PATH", request.param)
+    return request.param
+
+
+@pytest.mark.parametrize("forced_path", ["kernels", "persistent"], indirect=True)
+@pytest.mark.parametrize("shape,S,V", [(SHAPE_A, 1, 3), (SHAPE_C, 1, 2)], ids=["A", "C"])
+def test_both_execution_paths(pkg, oracle_mod, forced_path, shape, S, V):
+    # the per-operation kernel chain and the persistent all-layers kernel give the same
+    # lists and tokens within tolerance (full encode, cold start and steady state)
+    w = synth.make_weights(shape, 25)
+    frames = list(synth.stream_random(shape, S * V, 4, 26, change_p=0.15))
+    run_side_by_side(pkg, oracle_mod, shape, w, frames, S, V, check_caches=True)
+    run_side_by_side(pkg, oracle_mod, shape, w, frames[:2], S, V, first_full=False)

@@ -91,3 +91,10 @@ def test_so400m_448_batched(pkg, oracle_mod):
     finally:
         enc.close()
         orc.close()
+
+
+def test_so400m_1view_prefix_persistent_path(pkg, oracle_mod, monkeypatch):
+    monkeypatch.setenv("IVIT_PATH", "persistent")
+    wl = synth.WORKLOADS["so400m_224_1view"]
+    w = synth.make_weights(wl.shape, 0)
+    run_side_by_side(pkg, oracle_mod, wl.shape, w, _frames(wl, 3), check_caches=True)
