@@ -26,6 +26,7 @@ struct LayerW {
   bf16 *wqkv, *wo, *w1, *w2;
   float *bqkv, *bo, *b1, *b2, *ln1g, *ln1b, *ln2g, *ln2b;
   CUtensorMap tm_qkv, tm_o, tm_1, tm_2;
+  CUtensorMap tm_ck, tm_cv;  // this layer's key / value cache, attention key-split tiles
 };
 
 struct EventPair {
@@ -471,6 +472,13 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   h->err = sa.at<int>(o_err);
   h->frames_buf = sa.at<uint8_t>(o_fb);
   h->counts_buf = sa.at<int>(o_cb);
+  const int kps = ivit::attention_keys_per_split(h->N);
+  for (size_t l = 0; l < L; ++l) {
+    const size_t off = l * M * D;
+    if (!make_map(&h->layers[l].tm_ck, h->cacheK + off, D, M, D * 2, D / h->H, kps, false) ||
+        !make_map(&h->layers[l].tm_cv, h->cacheV + off, D, M, D * 2, D / h->H, kps, false))
+      return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for a cache tile");
+  }
   if (!make_map(&h->tm_patches, h->patches, h->KPAD, M, h->KPAD * 2, 64, 32) ||
       !make_map(&h->tm_xn, h->xn, D, M, D * 2, 64, 32) ||
       !make_map(&h->tm_o, h->o, D, M, D * 2, 64, 32) ||
@@ -625,7 +633,8 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
       a.epi.dim = D;
       if (int r = gemm(h, plan[kGemmQKV], w.tm_qkv, h->tm_xn, a, s)) return r;
     }
-    IVIT_CK(h, ivit::launch_attention(h->q, ck, cv, h->cu_rows, h->rowtok, h->o, SV, N, D, h->H, s));
+    IVIT_CK(h, ivit::launch_attention(w.tm_ck, w.tm_cv, h->q, ck, cv, h->cu_rows, h->rowtok, h->o, SV, N, D, h->H,
+                                      full ? (N + 31) / 32 : std::max(1, (N / 10 + 31) / 32), s));
     ++h->launches;
     {
       ivit::GemmArgs a;

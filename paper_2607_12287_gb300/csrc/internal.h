@@ -149,10 +149,16 @@ cudaError_t attention_setup();
 
 // O[r] = softmax(Q[r] K_v^T / sqrt(dh)) V_v per head, for the packed query rows r of
 // each view v (cu_rows), over the N cached keys/values of that view.
-// rowtok lists the updated tokens (packed row -> v*N + i): their keys are re-read after
-// the wait on the QKV kernel, every other key may be read before it.
-cudaError_t launch_attention(const bf16* q, const bf16* cache_k, const bf16* cache_v,
-                             const int* cu_rows, const int* rowtok, bf16* o, int sv, int n_tok,
-                             int dim, int heads, cudaStream_t s);
+// Keys per CTA of the attention kernel for N tokens per view (the key-split width).
+int attention_keys_per_split(int n_tok);
+// tm_k / tm_v: this layer's key / value cache, bf16 [SV*N][D], box [kps rows][dh], no
+// swizzle.  rowtok lists the updated tokens (packed row -> v*N + i): their keys are
+// re-read after the wait on the QKV kernel, every other key is loaded before it.
+// query_blocks: clusters per (view, head) along the queries (each loops over blocks of
+// 32 queries with its key tile resident); any value is correct, it sets parallelism.
+cudaError_t launch_attention(const CUtensorMap& tm_k, const CUtensorMap& tm_v, const bf16* q,
+                             const bf16* cache_k, const bf16* cache_v, const int* cu_rows,
+                             const int* rowtok, bf16* o, int sv, int n_tok, int dim, int heads,
+                             int query_blocks, cudaStream_t s);
 
 }  // namespace ivit

@@ -261,71 +261,57 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, const float* __r
 // K/V with this call's updated rows already written), per head:
 //   O = softmax(Q K^T / sqrt(dh)) V.
 // Grid: (query block x key split, head, view); the key splits of one query block form
-// a thread-block cluster.  Each CTA keeps its whole key range (at most ATT_KR keys) in
-// shared memory as bf16, K transposed so lanes read consecutive keys.  The range is
-// loaded before waiting on the QKV kernel (the cached keys of reused tokens do not
-// change), and only the keys of this call's updated tokens are read again after it.
-// Per query: online softmax over 64-key sub-tiles (running max m, sum l, output row in
-// registers), then the cluster merges its partial (m, l, o) through distributed
-// shared memory:  M = max_s m_s,  O = sum_s exp(m_s - M) o_s / sum_s exp(m_s - M) l_s.
-// Warp w owns queries 4w..4w+3; lane owns keys lane, lane+32 of a sub-tile for the
-// scores and output dims lane + 32c for P V.
+// a thread-block cluster.  Each CTA brings its key range (kps <= 128 keys) of K and V
+// into shared memory with one TMA load each, [keys][dh] bf16, issued before waiting on
+// the QKV kernel (the cached keys of reused tokens do not change); after the wait it
+// re-reads only the keys of this call's updated tokens.  Warp w owns queries
+// 4w..4w+3: scores with lanes owning keys (16-byte row loads), softmax in fp32 over the
+// CTA's keys, P V with lanes owning output dims; the cluster then merges its partial
+// (m, l, o) through distributed shared memory:
+//   M = max_s m_s,  O = sum_s exp(m_s - M) o_s / sum_s exp(m_s - M) l_s.
 constexpr int ATT_WARPS = 8;
 constexpr int ATT_QPW = 4;
 constexpr int ATT_QB = ATT_WARPS * ATT_QPW;
-constexpr int ATT_KT = 64;    // keys per softmax sub-tile
 constexpr int ATT_KR = 128;   // max keys per CTA (key split)
 
-__device__ __forceinline__ void att_store_key(bf16* skT, bf16* sv, int dh, int j, int c, uint4 uk,
-                                              uint4 uv) {
-  const bf16* k8 = reinterpret_cast<const bf16*>(&uk);
-#pragma unroll
-  for (int i = 0; i < 8; ++i) skT[(c * 8 + i) * ATT_KR + j] = k8[i];
-  *reinterpret_cast<uint4*>(sv + j * dh + c * 8) = uv;
-}
-
 __global__ void __launch_bounds__(ATT_WARPS * 32)
-    attention_kernel(const bf16* __restrict__ q, const bf16* __restrict__ cache_k,
+    attention_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                     const bf16* __restrict__ q, const bf16* __restrict__ cache_k,
                      const bf16* __restrict__ cache_v, const int* __restrict__ cu_rows,
-                     const int* __restrict__ rowtok, bf16* __restrict__ o, int N, int dim, int dh,
-                     int keys_per_split) {
-  extern __shared__ float sm[];
-  float* sq = sm;                                   // [QB][dh] fp32, pre-scaled
-  float* sp = sq + ATT_QB * dh;                     // [WARPS][QPW][KT]
-  float* sml = sp + ATT_WARPS * ATT_QPW * ATT_KT;   // [QB][2]
-  float* so = sml + 2 * ATT_QB;                     // [QB][dh] partial outputs
-  bf16* skT = reinterpret_cast<bf16*>(so + ATT_QB * dh);  // [dh][KR]
-  bf16* sv = skT + dh * ATT_KR;                           // [KR][dh]
+                     const int* __restrict__ rowtok, bf16* __restrict__ o, int N, int dim, int dh, int kps) {
+  extern __shared__ __align__(128) uint8_t att_smem[];
+  bf16* sk = reinterpret_cast<bf16*>(att_smem);            // [kps][dh]
+  bf16* sv = sk + ATT_KR * dh;                              // [kps][dh]
+  float* sq = reinterpret_cast<float*>(sv + ATT_KR * dh);   // [QB][dh] (later: partial o)
+  float* sp = sq + ATT_QB * dh;                             // [WARPS][QPW][KR]
+  float* sml = sp + ATT_WARPS * ATT_QPW * ATT_KR;           // [QB][2]
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sml + 2 * ATT_QB);
   const int ns = static_cast<int>(cluster_nctarank());
   const int rank = static_cast<int>(cluster_ctarank());
-  const int v = blockIdx.z, h = blockIdx.y, qb = blockIdx.x / ns;
+  const int v = blockIdx.z, h = blockIdx.y;
+  const int qb_first = blockIdx.x / ns, qb_stride = gridDim.x / ns;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int dh8 = dh / 8;
   // Row ranges come from the selection kernel (complete before this grid can start).
   const int r_begin = cu_rows[v], r_end = cu_rows[v + 1];
-  const int q0 = r_begin + qb * ATT_QB;
-  if (q0 >= r_end) {  // the whole cluster shares qb, so it leaves together
-    pdl_wait();
-    pdl_launch_dependents();
-    return;
-  }
-  const int nq = min(ATT_QB, r_end - q0);
-  const int k_begin = rank * keys_per_split, k_end = min(N, k_begin + keys_per_split);
-  const int nkr = k_end - k_begin;
+  if (r_begin + qb_first * ATT_QB >= r_end) return;  // the whole cluster leaves together
+  const int k_begin = rank * kps, nkr = min(N, k_begin + kps) - k_begin;
   const size_t vbase = static_cast<size_t>(v) * N;
-
-  // cached keys/values of the range (reused tokens' rows are final already)
-  for (int e = tid; e < ATT_KR * dh8; e += blockDim.x) {
-    const int j = e % ATT_KR, c = e / ATT_KR;
-    if (j < nkr) {
-      const size_t g = (vbase + k_begin + j) * dim + h * dh + c * 8;
-      att_store_key(skT, sv, dh, j, c, *reinterpret_cast<const uint4*>(cache_k + g),
-                    *reinterpret_cast<const uint4*>(cache_v + g));
-    }
+  const uint32_t bar_addr = smem_u32(bar);
+  bool ok = true;
+  if (tid == 0) {
+    mbar_init(bar_addr, 1);
+    fence_mbar_init();
+    const uint32_t bytes = static_cast<uint32_t>(kps) * dh * 2;
+    mbar_arrive_expect_tx(bar_addr, 2 * bytes);
+    tma_load_2d(smem_u32(sk), &tm_k, h * dh, static_cast<int>(vbase) + k_begin, bar_addr, l2_policy_evict_first());
+    tma_load_2d(smem_u32(sv), &tm_v, h * dh, static_cast<int>(vbase) + k_begin, bar_addr, l2_policy_evict_first());
   }
+  __syncthreads();  // barrier initialised before anyone waits on it
   pdl_wait();  // the QKV kernel's queries and new K/V rows are visible from here
   pdl_launch_dependents();
-
+  if (!mbar_wait(bar_addr, 0)) ok = false;  // (all threads) cached tile landed
+  __syncthreads();
   // re-read the keys this call updated (tokens of view v listed in rowtok)
   const int n_upd = r_end - r_begin;
   for (int e = tid; e < n_upd * dh8; e += blockDim.x) {
@@ -333,24 +319,29 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
     const int j = rowtok[r_begin + r] - static_cast<int>(vbase) - k_begin;
     if (j >= 0 && j < nkr) {
       const size_t g = (vbase + k_begin + j) * dim + h * dh + c * 8;
-      att_store_key(skT, sv, dh, j, c, __ldcg(reinterpret_cast<const uint4*>(cache_k + g)),
-                    __ldcg(reinterpret_cast<const uint4*>(cache_v + g)));
+      *reinterpret_cast<uint4*>(sk + j * dh + c * 8) = __ldcg(reinterpret_cast<const uint4*>(cache_k + g));
+      *reinterpret_cast<uint4*>(sv + j * dh + c * 8) = __ldcg(reinterpret_cast<const uint4*>(cache_v + g));
     }
   }
   const float scale = rsqrtf(static_cast<float>(dh));
+  // query blocks of this view handled by this cluster (the key tile stays resident)
+  for (int qb = qb_first; r_begin + qb * ATT_QB < r_end; qb += qb_stride) {
+  const int q0 = r_begin + qb * ATT_QB;
+  const int nq = min(ATT_QB, r_end - q0);
+  __syncthreads();  // previous block's queries and partials are consumed
   for (int e = tid; e < nq * dh8; e += blockDim.x) {
     const int qi = e / dh8, c = e % dh8;
     const uint4 u = __ldcg(reinterpret_cast<const uint4*>(q + static_cast<size_t>(q0 + qi) * dim + h * dh + c * 8));
     const __nv_bfloat162* b2 = reinterpret_cast<const __nv_bfloat162*>(&u);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float2 f = __bfloat1622float2(b2[i]);
-      sq[qi * dh + c * 8 + 2 * i] = f.x * scale;
-      sq[qi * dh + c * 8 + 2 * i + 1] = f.y * scale;
-    }
+    float4* dst = reinterpret_cast<float4*>(sq + qi * dh + c * 8);
+    const float2 f0 = __bfloat1622float2(b2[0]), f1 = __bfloat1622float2(b2[1]);
+    const float2 f2 = __bfloat1622float2(b2[2]), f3 = __bfloat1622float2(b2[3]);
+    dst[0] = make_float4(f0.x * scale, f0.y * scale, f1.x * scale, f1.y * scale);
+    dst[1] = make_float4(f2.x * scale, f2.y * scale, f3.x * scale, f3.y * scale);
   }
   __syncthreads();
 
+  const int qa = warp * ATT_QPW;
   float m_run[ATT_QPW], l_run[ATT_QPW], acc[ATT_QPW][4];
 #pragma unroll
   for (int a = 0; a < ATT_QPW; ++a) {
@@ -359,60 +350,81 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc[a][c] = 0.f;
   }
-  float* spw = sp + warp * ATT_QPW * ATT_KT;
-  const float* qw = sq + warp * ATT_QPW * dh;
-  const bool warp_active = warp * ATT_QPW < nq;
-
-  for (int t0 = 0; t0 < nkr && warp_active; t0 += ATT_KT) {
-    const int nk = min(ATT_KT, nkr - t0);
-    float s0[ATT_QPW], s1[ATT_QPW];
+  if (qa < nq && ok) {
+    float* spw = sp + warp * ATT_QPW * ATT_KR;
+    // scores: lane owns keys lane + 32 kk of the CTA's range
+    float sc[ATT_QPW][4];
 #pragma unroll
-    for (int a = 0; a < ATT_QPW; ++a) s0[a] = s1[a] = 0.f;
-    for (int d = 0; d < dh; ++d) {
-      const float k0v = __bfloat162float(skT[d * ATT_KR + t0 + lane]);
-      const float k1v = __bfloat162float(skT[d * ATT_KR + t0 + lane + 32]);
+    for (int a = 0; a < ATT_QPW; ++a)
 #pragma unroll
-      for (int a = 0; a < ATT_QPW; ++a) {
-        const float qv = qw[a * dh + d];
-        s0[a] += qv * k0v;
-        s1[a] += qv * k1v;
+      for (int kk = 0; kk < 4; ++kk) sc[a][kk] = 0.f;
+    for (int d = 0; d < dh; d += 8) {
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        const int j = lane + 32 * kk;
+        if (j < nkr) {
+          const uint4 raw = *reinterpret_cast<const uint4*>(sk + j * dh + d);
+          const __nv_bfloat162* k2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
+          const float2 f0 = __bfloat1622float2(k2[0]), f1 = __bfloat1622float2(k2[1]);
+          const float2 f2 = __bfloat1622float2(k2[2]), f3 = __bfloat1622float2(k2[3]);
+#pragma unroll
+          for (int a = 0; a < ATT_QPW; ++a) {
+            const float4 lo = *reinterpret_cast<const float4*>(sq + (qa + a) * dh + d);
+            const float4 hi = *reinterpret_cast<const float4*>(sq + (qa + a) * dh + d + 4);
+            sc[a][kk] += lo.x * f0.x + lo.y * f0.y + lo.z * f1.x + lo.w * f1.y + hi.x * f2.x + hi.y * f2.y +
+                         hi.z * f3.x + hi.w * f3.y;
+          }
+        }
       }
     }
 #pragma unroll
     for (int a = 0; a < ATT_QPW; ++a) {
-      const float x0 = lane < nk ? s0[a] : -INFINITY;
-      const float x1 = lane + 32 < nk ? s1[a] : -INFINITY;
-      const float m_new = fmaxf(m_run[a], warp_max(fmaxf(x0, x1)));
-      const float corr = __expf(m_run[a] - m_new);
-      const float p0 = lane < nk ? __expf(x0 - m_new) : 0.f;
-      const float p1 = lane + 32 < nk ? __expf(x1 - m_new) : 0.f;
-      l_run[a] = l_run[a] * corr + warp_sum(p0 + p1);
-      m_run[a] = m_new;
+      float mx = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) acc[a][c] *= corr;
-      spw[a * ATT_KT + lane] = p0;
-      spw[a * ATT_KT + lane + 32] = p1;
-    }
-    __syncwarp();
-    for (int j = 0; j < nk; ++j) {
-      float vv[4];
+      for (int kk = 0; kk < 4; ++kk)
+        if (lane + 32 * kk < nkr) mx = fmaxf(mx, sc[a][kk]);
+      mx = warp_max(mx);
+      float sum = 0.f;
 #pragma unroll
-      for (int c = 0; c < 4; ++c)
-        vv[c] = (lane + 32 * c < dh) ? __bfloat162float(sv[(t0 + j) * dh + lane + 32 * c]) : 0.f;
-#pragma unroll
-      for (int a = 0; a < ATT_QPW; ++a) {
-        const float pj = spw[a * ATT_KT + j];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) acc[a][c] += pj * vv[c];
+      for (int kk = 0; kk < 4; ++kk) {
+        const int j = lane + 32 * kk;
+        if (j < nkr) {
+          const float p = __expf(sc[a][kk] - mx);
+          spw[a * ATT_KR + j] = p;
+          sum += p;
+        }
       }
+      m_run[a] = mx;
+      l_run[a] = warp_sum(sum);
     }
     __syncwarp();
+    // P V: lanes own dims lane + 32 c; 8 keys per step with every load issued first
+    for (int j0 = 0; j0 < nkr; j0 += 8) {
+      float pk[ATT_QPW][8], vk[8][4];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int j = j0 + u;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const int d = lane + 32 * c;
+          vk[u][c] = (j < nkr && d < dh) ? __bfloat162float(sv[j * dh + d]) : 0.f;
+        }
+#pragma unroll
+        for (int a = 0; a < ATT_QPW; ++a) pk[a][u] = j < nkr ? spw[a * ATT_KR + j] : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+#pragma unroll
+        for (int a = 0; a < ATT_QPW; ++a)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[a][c] += pk[a][u] * vk[u][c];
+    }
   }
 
   if (ns == 1) {
 #pragma unroll
     for (int a = 0; a < ATT_QPW; ++a) {
-      const int qi = warp * ATT_QPW + a;
+      const int qi = qa + a;
       if (qi < nq) {
         const float inv = 1.f / l_run[a];
         bf16* orow = o + static_cast<size_t>(q0 + qi) * dim + h * dh;
@@ -421,13 +433,15 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
           if (lane + 32 * c < dh) orow[lane + 32 * c] = __float2bfloat16_rn(acc[a][c] * inv);
       }
     }
-    return;
+    continue;
   }
 
   // partial (m, l, o) of every query of the block, then a cluster-wide merge
+  __syncthreads();  // every warp is done with sq
+  float* so = sq;
 #pragma unroll
   for (int a = 0; a < ATT_QPW; ++a) {
-    const int qi = warp * ATT_QPW + a;
+    const int qi = qa + a;
 #pragma unroll
     for (int c = 0; c < 4; ++c)
       if (lane + 32 * c < dh) so[qi * dh + lane + 32 * c] = acc[a][c];
@@ -440,15 +454,15 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
   const uint32_t so_addr = smem_u32(so), ml_addr = smem_u32(sml);
   for (int qi = rank + ns * warp; qi < nq; qi += ns * ATT_WARPS) {
     float M = -INFINITY;
-    for (int s = 0; s < ns; ++s) M = fmaxf(M, ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi, s)));
+    for (int s2 = 0; s2 < ns; ++s2) M = fmaxf(M, ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi, s2)));
     float lsum = 0.f, out[4] = {0.f, 0.f, 0.f, 0.f};
-    for (int s = 0; s < ns; ++s) {
-      const float w = __expf(ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi, s)) - M);
-      lsum += w * ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi + 4, s));
+    for (int s2 = 0; s2 < ns; ++s2) {
+      const float w = __expf(ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi, s2)) - M);
+      lsum += w * ld_dsmem_f32(mapa_shared(ml_addr + 8 * qi + 4, s2));
 #pragma unroll
       for (int c = 0; c < 4; ++c)
         if (lane + 32 * c < dh)
-          out[c] += w * ld_dsmem_f32(mapa_shared(so_addr + 4 * (qi * dh + lane + 32 * c), s));
+          out[c] += w * ld_dsmem_f32(mapa_shared(so_addr + 4 * (qi * dh + lane + 32 * c), s2));
     }
     const float inv = 1.f / lsum;
     bf16* orow = o + static_cast<size_t>(q0 + qi) * dim + h * dh;
@@ -457,6 +471,7 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
       if (lane + 32 * c < dh) orow[lane + 32 * c] = __float2bfloat16_rn(out[c] * inv);
   }
   cluster_sync();  // partials stay valid until every CTA of the cluster has read them
+  }  // query blocks
 }
 
 }  // namespace
@@ -501,8 +516,14 @@ cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma
 }
 
 size_t attention_smem(int dh) {
-  return (2 * ATT_QB * dh + ATT_WARPS * ATT_QPW * ATT_KT + 2 * ATT_QB) * sizeof(float) +
-         2 * static_cast<size_t>(dh) * ATT_KR * sizeof(bf16);
+  return 2 * static_cast<size_t>(ATT_KR) * dh * sizeof(bf16) +
+         (ATT_QB * dh + ATT_WARPS * ATT_QPW * ATT_KR + 2 * ATT_QB) * sizeof(float) + 16;
+}
+
+int attention_keys_per_split(int n_tok) {
+  int ns = (n_tok + 63) / 64;  // key splits of about 64 keys, at most 8 (portable cluster)
+  ns = ns < 1 ? 1 : (ns > 8 ? 8 : ns);
+  return (n_tok + ns - 1) / ns;
 }
 
 cudaError_t attention_setup() {
@@ -510,17 +531,19 @@ cudaError_t attention_setup() {
                               static_cast<int>(attention_smem(128)));
 }
 
-cudaError_t launch_attention(const bf16* q, const bf16* cache_k, const bf16* cache_v,
-                             const int* cu_rows, const int* rowtok, bf16* o, int sv, int n_tok,
-                             int dim, int heads, cudaStream_t s) {
+cudaError_t launch_attention(const CUtensorMap& tm_k, const CUtensorMap& tm_v, const bf16* q,
+                             const bf16* cache_k, const bf16* cache_v, const int* cu_rows,
+                             const int* rowtok, bf16* o, int sv, int n_tok, int dim, int heads,
+                             int query_blocks, cudaStream_t s) {
   const int dh = dim / heads;
-  // key splits of about 64 keys (at most 128, at most 8 CTAs: a portable cluster)
-  int ns = (n_tok + ATT_KT - 1) / ATT_KT;
-  ns = ns < 1 ? 1 : (ns > 8 ? 8 : ns);
-  const int kps = (n_tok + ns - 1) / ns;
-  const dim3 grid(((n_tok + ATT_QB - 1) / ATT_QB) * ns, heads, sv);
+  const int kps = attention_keys_per_split(n_tok);
+  const int ns = (n_tok + kps - 1) / kps;
+  const int max_qb = (n_tok + ATT_QB - 1) / ATT_QB;
+  const int qbs = query_blocks < 1 ? 1 : (query_blocks > max_qb ? max_qb : query_blocks);
+  const dim3 grid(qbs * ns, heads, sv);
   return launch_ex(attention_kernel, grid, dim3(ATT_WARPS * 32), attention_smem(dh), s,
-                   static_cast<unsigned>(ns), q, cache_k, cache_v, cu_rows, rowtok, o, n_tok, dim, dh, kps);
+                   static_cast<unsigned>(ns), tm_k, tm_v, q, cache_k, cache_v, cu_rows, rowtok, o, n_tok, dim,
+                   dh, kps);
 }
 
 }  // namespace ivit
