@@ -19,6 +19,8 @@ _HDR = os.path.join(_HERE, "ivit_oracle.h")
 _LIB = os.path.join(_HERE, "_build", "liboracle.so")
 
 GELU_TANH, GELU_ERF = 0, 1
+SCORE_EMBED, SCORE_KEY0 = 0, 1
+SCHED_INCREMENTAL, SCHED_ODD_EVEN = 0, 1
 SEL_THRESHOLD, SEL_TOPK = 0, 1
 REF_PREV_FRAME, REF_LAST_REFRESH = 0, 1
 
@@ -30,6 +32,7 @@ class OrcConfig(C.Structure):
         ("mlp_dim", C.c_int32), ("n_streams", C.c_int32), ("n_views", C.c_int32),
         ("ln_eps", C.c_float), ("gelu", C.c_int32), ("select_mode", C.c_int32),
         ("threshold", C.c_float), ("topk", C.c_int32), ("ref_mode", C.c_int32),
+        ("score_source", C.c_int32), ("schedule", C.c_int32),
     ]
 
 
@@ -73,6 +76,7 @@ def lib() -> C.CDLL:
         L.orc_gelu.argtypes = [C.c_float, C.c_int]
         L.orc_attention.argtypes = [P, C.c_int, P, P, C.c_int, C.c_int, C.c_int, C.c_int,
                                     P, C.c_int]
+        L.orc_layer0_keys.argtypes = [P, P, P, P, P, P, C.c_int, C.c_int, C.c_float, P]
         _lib = L
     return _lib
 
@@ -90,10 +94,11 @@ def set_threads(n: int) -> None:
 
 
 def make_config(shape, n_streams=1, n_views=1, select_mode=SEL_THRESHOLD, threshold=0.98,
-                topk=0, ref_mode=REF_PREV_FRAME) -> OrcConfig:
+                topk=0, ref_mode=REF_PREV_FRAME, score_source=SCORE_EMBED,
+                schedule=SCHED_INCREMENTAL) -> OrcConfig:
     return OrcConfig(shape.img_h, shape.img_w, shape.patch, shape.dim, shape.depth,
                      shape.heads, shape.mlp_dim, n_streams, n_views, shape.ln_eps,
-                     shape.gelu, select_mode, threshold, topk, ref_mode)
+                     shape.gelu, select_mode, threshold, topk, ref_mode, score_source, schedule)
 
 
 class Oracle:
@@ -101,10 +106,10 @@ class Oracle:
 
     def __init__(self, shape, weights_u16: np.ndarray, n_streams=1, n_views=1,
                  select_mode=SEL_THRESHOLD, threshold=0.98, topk=0,
-                 ref_mode=REF_PREV_FRAME):
+                 ref_mode=REF_PREV_FRAME, score_source=SCORE_EMBED, schedule=SCHED_INCREMENTAL):
         self.shape = shape
         self.cfg = make_config(shape, n_streams, n_views, select_mode, threshold, topk,
-                               ref_mode)
+                               ref_mode, score_source, schedule)
         self.sv = n_streams * n_views
         self._w = np.ascontiguousarray(weights_u16, dtype=np.uint16)
         self._h = lib().orc_create(C.byref(self.cfg), _p(self._w))
@@ -114,7 +119,7 @@ class Oracle:
     @classmethod
     def for_workload(cls, wl, weights_u16):
         return cls(wl.shape, weights_u16, wl.n_streams, wl.n_views, wl.select_mode,
-                   wl.threshold, wl.topk, wl.ref_mode)
+                   wl.threshold, wl.topk, wl.ref_mode, wl.score_source, wl.schedule)
 
     def close(self):
         if self._h:
@@ -208,6 +213,14 @@ def linear(x, W, b) -> np.ndarray:
 
 def gelu(x: float, mode: int) -> float:
     return float(lib().orc_gelu(float(x), int(mode)))
+
+
+def layer0_keys(e, pos, ln_g, ln_b, W_K, b_K, eps: float = 1e-6) -> np.ndarray:
+    e, pos, g, b, W, bk = (_f32(a) for a in (e, pos, ln_g, ln_b, W_K, b_K))
+    n, D = e.shape
+    k = np.empty((n, D), np.float32)
+    lib().orc_layer0_keys(_p(e), _p(pos), _p(g), _p(b), _p(W), _p(bk), n, D, float(eps), _p(k))
+    return k
 
 
 def attention(q, k, v) -> np.ndarray:

@@ -14,8 +14,9 @@
  *   - attention computed for the updated tokens only, which attend over all tokens;
  *     reused tokens keep their cached outputs (Sec. III-B).
  * Readings where the paper is silent are listed in the repository's design notes:
- * the score compares patch embeddings (before the position embedding) with the
- * previous frame; all updated tokens' K/V of a layer are written before that layer's
+ * the score compares either the patch embeddings (before the position embedding) or
+ * the first layer's keys (Eq. 3 as printed) with their reference; all updated tokens'
+ * K/V of a layer are written before that layer's
  * attention; reused tokens' residual streams are never touched; the cached output is
  * the post-final-LN token; a cold view (no reference yet) updates every token.
  *
@@ -44,8 +45,10 @@ struct orc_state {
   float* wbuf;
   const float *W_pe, *b_pe, *pos, *lnf_g, *lnf_b;
   orc_layer* layer;
-  float* e_ref;   /* [SV][N][D] */
+  float* e_ref;   /* [SV][N][D] reference score vectors */
   float* e_t;     /* [SV][N][D] scratch: this frame's patch embeddings */
+  float* s_t;     /* [SV][N][D] scratch: this frame's score vectors (first-layer keys) */
+  long long chunk; /* incremental calls made (odd/even schedule) */
   float* cacheK;  /* [L][SV][N][D] */
   float* cacheV;  /* [L][SV][N][D] */
   float* tok_out; /* [SV][N][D] final tokens (post final LN) */
@@ -147,6 +150,30 @@ float orc_gelu(float x, int mode) {
   if (mode == 1) return (float)(0.5 * xd * (1.0 + erf(xd / sqrt(2.0))));
   const double c = sqrt(2.0 / M_PI);
   return (float)(0.5 * xd * (1.0 + tanh(c * (xd + 0.044715 * xd * xd * xd))));
+}
+
+static float round_bf16(float x) {
+  uint32_t u;
+  memcpy(&u, &x, sizeof u);
+  u = (u + 0x7FFFu + ((u >> 16) & 1u)) & 0xFFFF0000u; /* nearest, ties to even */
+  float y;
+  memcpy(&y, &u, sizeof y);
+  return y;
+}
+
+void orc_layer0_keys(const float* e, const float* pos, const float* ln_g, const float* ln_b,
+                     const float* W_K, const float* b_K, int n, int D, float eps, float* k) {
+#pragma omp parallel for schedule(static)
+  for (int i = 0; i < n; ++i) {
+    float* x = (float*)malloc(sizeof(float) * (size_t)D);
+    float* xn = (float*)malloc(sizeof(float) * (size_t)D);
+    for (int d = 0; d < D; ++d) x[d] = e[(size_t)i * D + d] + pos[(size_t)i * D + d];
+    orc_layernorm(x, ln_g, ln_b, D, eps, xn);
+    for (int d = 0; d < D; ++d) xn[d] = round_bf16(xn[d]);
+    orc_linear(xn, W_K, b_K, D, D, k + (size_t)i * D);
+    free(x);
+    free(xn);
+  }
 }
 
 static void attention_row(const float* q, const float* k, const float* v, int kv_stride,
@@ -315,11 +342,12 @@ orc_state* orc_create(const orc_config* cfg, const uint16_t* wb) {
   const size_t view = (size_t)s->SV * N * D;
   s->e_ref = (float*)calloc(view, sizeof(float));
   s->e_t = (float*)calloc(view, sizeof(float));
+  s->s_t = (float*)calloc(view, sizeof(float));
   s->tok_out = (float*)calloc(view, sizeof(float));
   s->cacheK = (float*)calloc(view * s->L, sizeof(float));
   s->cacheV = (float*)calloc(view * s->L, sizeof(float));
   s->cold = (uint8_t*)malloc((size_t)s->SV);
-  if (!s->e_ref || !s->e_t || !s->tok_out || !s->cacheK || !s->cacheV || !s->cold) {
+  if (!s->e_ref || !s->e_t || !s->s_t || !s->tok_out || !s->cacheK || !s->cacheV || !s->cold) {
     orc_destroy(s);
     return NULL;
   }
@@ -333,6 +361,7 @@ void orc_destroy(orc_state* s) {
   free(s->layer);
   free(s->e_ref);
   free(s->e_t);
+  free(s->s_t);
   free(s->tok_out);
   free(s->cacheK);
   free(s->cacheV);
@@ -340,11 +369,22 @@ void orc_destroy(orc_state* s) {
   free(s);
 }
 
+/* Patch embeddings of every view, and the score vectors Eq. 3 compares: the
+ * embeddings themselves, or the first layer's keys of every token. */
 static void embed_all(orc_state* s, const uint8_t* frames) {
   const size_t frame_bytes = (size_t)s->cfg.img_h * s->cfg.img_w * 3;
-  for (int v = 0; v < s->SV; ++v)
-    orc_patch_embed(&s->cfg, s->W_pe, s->b_pe, frames + (size_t)v * frame_bytes,
-                    s->e_t + (size_t)v * s->N * s->D);
+  const size_t D = s->D;
+  for (int v = 0; v < s->SV; ++v) {
+    float* e = s->e_t + (size_t)v * s->N * D;
+    orc_patch_embed(&s->cfg, s->W_pe, s->b_pe, frames + (size_t)v * frame_bytes, e);
+    if (s->cfg.score_source == 1)
+      orc_layer0_keys(e, s->pos, s->layer[0].ln1_g, s->layer[0].ln1_b, s->layer[0].W_qkv + D * D,
+                      s->layer[0].b_qkv + D, s->N, s->D, s->cfg.ln_eps, s->s_t + (size_t)v * s->N * D);
+  }
+}
+
+static const float* score_vectors(const orc_state* s) {
+  return s->cfg.score_source == 1 ? s->s_t : s->e_t;
 }
 
 static void copy_out(const orc_state* s, float* tokens_out) {
@@ -359,7 +399,7 @@ int orc_encode_full(orc_state* s, const uint8_t* frames, float* tokens_out) {
   int32_t* U = (int32_t*)malloc(sizeof(int32_t) * (size_t)N);
   for (int i = 0; i < N; ++i) U[i] = i;
   for (int v = 0; v < s->SV; ++v) {
-    memcpy(s->e_ref + (size_t)v * N * D, s->e_t + (size_t)v * N * D,
+    memcpy(s->e_ref + (size_t)v * N * D, score_vectors(s) + (size_t)v * N * D,
            sizeof(float) * (size_t)N * D);
     encode_rows(s, v, U, N);
     s->cold[v] = 0;
@@ -373,11 +413,23 @@ int orc_encode_incremental(orc_state* s, const uint8_t* frames, float* tokens_ou
                            int32_t* counts_out, int32_t* idx_out, float* sims_out) {
   if (!s || !frames) return -1;
   const int N = s->N, D = s->D;
+  /* odd/even schedule: odd chunks (1st, 3rd, ... call) encode every token in full */
+  if (s->cfg.schedule == 1 && (s->chunk++ % 2) == 0) {
+    orc_encode_full(s, frames, tokens_out);
+    for (int v = 0; v < s->SV; ++v) {
+      if (counts_out) counts_out[v] = N;
+      if (idx_out)
+        for (int i = 0; i < N; ++i) idx_out[(size_t)v * N + i] = i;
+      if (sims_out)
+        for (int i = 0; i < N; ++i) sims_out[(size_t)v * N + i] = -2.f;
+    }
+    return 0;
+  }
   embed_all(s, frames);
   int32_t* U = (int32_t*)malloc(sizeof(int32_t) * (size_t)N);
   float* sims = (float*)malloc(sizeof(float) * (size_t)N);
   for (int v = 0; v < s->SV; ++v) {
-    const float* et = s->e_t + (size_t)v * N * D;
+    const float* et = score_vectors(s) + (size_t)v * N * D;
     float* er = s->e_ref + (size_t)v * N * D;
     int m;
     if (s->cold[v]) {

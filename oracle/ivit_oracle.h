@@ -35,6 +35,10 @@ typedef struct orc_config {
   float threshold;
   int32_t topk;
   int32_t ref_mode;    /* 0: reference = previous frame, 1: reference = last refresh */
+  int32_t score_source; /* 0: patch embeddings (before the position embedding),
+                           1: first-layer keys (Eq. 3) */
+  int32_t schedule;     /* 0: every incremental call is incremental,
+                           1: odd/even chunks (odd calls encode in full, Sec. III-B) */
 } orc_config;
 
 typedef struct orc_state orc_state;
@@ -59,7 +63,8 @@ int orc_encode_incremental(orc_state* s, const uint8_t* frames, float* tokens_ou
 int orc_reset(orc_state* s, int stream);
 
 /* Cache read-out for tests.  which: 0 = K, 1 = V (layer `layer`), 2 = final tokens,
- * 3 = reference embedding.  out: float [S*V][N][D]. */
+ * 3 = reference score vectors (patch embeddings or first-layer keys, per
+ * score_source).  out: float [S*V][N][D]. */
 int orc_get_cache(const orc_state* s, int which, int layer, float* out);
 
 /* ---- building blocks (each a step of the method, exported for pinning) ---- */
@@ -80,6 +85,11 @@ void orc_layernorm(const float* x, const float* g, const float* b, int n, float 
 void orc_linear(const float* x, const float* W, const float* b, int n_in, int n_out,
                 float* y);
 float orc_gelu(float x, int mode);
+/* Eq. 3 key vectors of the first layer for n tokens: k[i] = W_K bf16(LN1(e[i] + pos[i]))
+ * + b_K, with the LN output rounded to bf16 (the precision the GPU path computes the
+ * keys in, so both sides take the selection decision alike).  W_K [D][D]. */
+void orc_layer0_keys(const float* e, const float* pos, const float* ln_g, const float* ln_b,
+                     const float* W_K, const float* b_K, int n, int D, float eps, float* k);
 /* One head: o[r] = softmax_j(<q[r], k[j]> / sqrt(dh)) v[j]; q [m][q_stride],
  * k, v [n][kv_stride], o [m][o_stride]; head width dh. */
 void orc_attention(const float* q, int q_stride, const float* k, const float* v,

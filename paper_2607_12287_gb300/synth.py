@@ -38,6 +38,10 @@ import numpy as np
 
 GELU_TANH = 0
 GELU_ERF = 1
+SCORE_EMBED = 0
+SCORE_KEY0 = 1
+SCHED_INCREMENTAL = 0
+SCHED_ODD_EVEN = 1
 SEL_THRESHOLD = 0
 SEL_TOPK = 1
 REF_PREV_FRAME = 0
@@ -373,6 +377,8 @@ class Workload:
     threshold: float = 0.98
     topk: int = 0
     ref_mode: int = REF_PREV_FRAME
+    score_source: int = SCORE_EMBED
+    schedule: int = SCHED_INCREMENTAL
     scene: str = "rects"
     views: Tuple[ViewScene, ...] = field(default_factory=tuple)
     repaint_k: int = 0
