@@ -334,6 +334,7 @@ def main() -> None:
         "full_encode_ms_per_step": full_ms / args.steps,
         "full_encode_frames_per_s": frames_total / (full_ms / 1e3),
         "speedup_vs_full": full_ms / inc_ms,
+        "odd_even_ms_per_step": 0.5 * (full_ms + inc_ms) / args.steps,  # Sec. III-B chunking
         "e2e": {"value": frames_total / (e2e_ms / 1e3), "unit": "frames/s",
                 "ms_per_step": e2e_ms / args.steps,
                 "h2d_bytes_per_step": int(frames[0].nbytes),

@@ -46,6 +46,10 @@ extern "C" {
 #define IVIT_SEL_TOPK 1        /* update the topk lowest sims, ties by lower index */
 #define IVIT_REF_PREV_FRAME 0  /* reference = previous frame's embeddings (all tokens) */
 #define IVIT_REF_LAST_REFRESH 1 /* reference of token i updated only when i is updated */
+#define IVIT_SCORE_EMBED 0     /* Eq. 3 on patch embeddings (before position embedding) */
+#define IVIT_SCORE_KEY0 1      /* Eq. 3 as printed: first-layer keys W_K LN1(e+pos) + b_K */
+#define IVIT_SCHED_INCREMENTAL 0 /* every ivit_encode_incremental call is incremental */
+#define IVIT_SCHED_ODD_EVEN 1  /* odd calls encode in full, even calls incrementally */
 
 /* Encoder + selection configuration.
  * Supported by the kernels: patch >= 1 dividing img_h and img_w; N <= 1024;
@@ -66,6 +70,8 @@ typedef struct ivit_config {
   float threshold;       /* IVIT_SEL_THRESHOLD: refresh where sim < threshold */
   int32_t topk;          /* IVIT_SEL_TOPK: tokens refreshed per view, clamped to [0, N] */
   int32_t ref_mode;      /* IVIT_REF_* */
+  int32_t score_source;  /* IVIT_SCORE_*: what Eq. 3's cosine compares (Sec. III-B) */
+  int32_t schedule;      /* IVIT_SCHED_*: odd/even chunking of Sec. III-B, or none */
 } ivit_config;
 
 typedef struct ivit_handle ivit_handle;
@@ -94,13 +100,15 @@ int ivit_create(const ivit_config* cfg, const uint16_t* weights_bf16_host,
 int ivit_encode_full(ivit_handle* h, const uint8_t* frames_dev, uint16_t* tokens_out_dev,
                      void* stream);
 
-/* Incremental encode (Sec. III-B, Eq. 3-5): scores every token's patch embedding
- * against its reference (cosine, fp32), selects the tokens to update per view, runs
+/* Incremental encode (Sec. III-B, Eq. 3-5): scores every token's patch embedding, or
+ * its first-layer key (score_source), against its reference (cosine, fp32), selects
+ * the tokens to update per view, runs
  * every block on those tokens only (their queries attend over all N tokens of the
  * view, the others' K/V come from the cache), and returns all tokens: updated ones
  * recomputed, the rest from the final-token cache.  A cold view updates every token.
  * tokens_out_dev: bf16 [SV][N][D] or NULL.  changed_count_dev: int32 [SV] number of
- * updated tokens per view, or NULL.  No host synchronisation happens inside. */
+ * updated tokens per view, or NULL.  No host synchronisation happens inside.  With
+ * schedule = IVIT_SCHED_ODD_EVEN the 1st, 3rd, ... call encodes in full (count N). */
 int ivit_encode_incremental(ivit_handle* h, const uint8_t* frames_dev,
                             uint16_t* tokens_out_dev, int32_t* changed_count_dev,
                             void* stream);
@@ -112,8 +120,9 @@ int ivit_get_changed(ivit_handle* h, int sv, int32_t* idx_dev, int32_t* count_de
                      void* stream);
 
 /* Copies per-view state for inspection: which = 0 key cache of `layer`, 1 value cache
- * of `layer`, 2 final-token cache (all bf16 [SV][N][D]), 3 reference embeddings
- * (fp32 [SV][N][D]).  dst_dev must hold that many bytes. */
+ * of `layer`, 2 final-token cache (all bf16 [SV][N][D]), 3 reference score vectors
+ * (patch embeddings or first-layer keys, fp32 [SV][N][D]).  dst_dev must hold that many
+ * bytes. */
 int ivit_get_cache(ivit_handle* h, int which, int layer, void* dst_dev, void* stream);
 
 /* Marks the views of camera stream `stream_index` (all streams if -1) cold: the next

@@ -41,6 +41,7 @@ class IvitConfig(C.Structure):
         ("mlp_dim", C.c_int32), ("n_streams", C.c_int32), ("n_views", C.c_int32),
         ("ln_eps", C.c_float), ("gelu", C.c_int32), ("select_mode", C.c_int32),
         ("threshold", C.c_float), ("topk", C.c_int32), ("ref_mode", C.c_int32),
+        ("score_source", C.c_int32), ("schedule", C.c_int32),
     ]
 
 
@@ -107,10 +108,11 @@ def _stream(stream) -> Optional[int]:
 
 def make_config(shape: "synth.EncoderShape", n_streams: int = 1, n_views: int = 1,
                 select_mode: int = synth.SEL_THRESHOLD, threshold: float = 0.98, topk: int = 0,
-                ref_mode: int = synth.REF_PREV_FRAME) -> IvitConfig:
+                ref_mode: int = synth.REF_PREV_FRAME, score_source: int = synth.SCORE_EMBED,
+                schedule: int = synth.SCHED_INCREMENTAL) -> IvitConfig:
     return IvitConfig(shape.img_h, shape.img_w, shape.patch, shape.dim, shape.depth, shape.heads,
                       shape.mlp_dim, n_streams, n_views, shape.ln_eps, shape.gelu, select_mode,
-                      threshold, topk, ref_mode)
+                      threshold, topk, ref_mode, score_source, schedule)
 
 
 # ------------------------------------------------------------- C entry points
@@ -196,19 +198,21 @@ class IncrementalViT:
 
     def __init__(self, shape: "synth.EncoderShape", weights_u16: np.ndarray, n_streams: int = 1,
                  n_views: int = 1, select_mode: int = synth.SEL_THRESHOLD,
-                 threshold: float = 0.98, topk: int = 0, ref_mode: int = synth.REF_PREV_FRAME):
+                 threshold: float = 0.98, topk: int = 0, ref_mode: int = synth.REF_PREV_FRAME,
+                 score_source: int = synth.SCORE_EMBED, schedule: int = synth.SCHED_INCREMENTAL):
         import torch
         self.torch = torch
         self.shape = shape
         self.sv = n_streams * n_views
-        self.cfg = make_config(shape, n_streams, n_views, select_mode, threshold, topk, ref_mode)
+        self.cfg = make_config(shape, n_streams, n_views, select_mode, threshold, topk, ref_mode,
+                               score_source, schedule)
         self.h = ivit_create(self.cfg, weights_u16)
         self.device = torch.device("cuda", torch.cuda.current_device())
 
     @classmethod
     def for_workload(cls, wl, weights_u16):
         return cls(wl.shape, weights_u16, wl.n_streams, wl.n_views, wl.select_mode, wl.threshold,
-                   wl.topk, wl.ref_mode)
+                   wl.topk, wl.ref_mode, wl.score_source, wl.schedule)
 
     def close(self):
         if getattr(self, "h", None):

@@ -114,6 +114,11 @@ struct ivit_handle {
 
   bf16* patches = nullptr;
   float *e_t = nullptr, *e_ref = nullptr, *sims = nullptr, *x = nullptr;
+  float* key_t = nullptr;          // first-layer keys of every token (score_source KEY0)
+  int* rowtok_all = nullptr;       // identity row -> token map, all SV*N rows
+  int* m_all = nullptr;            // device copy of SV*N
+  CUtensorMap tm_wk0;              // layer 0's key projection (rows D..2D-1 of W_qkv)
+  long long chunk = 0;             // ivit_encode_incremental calls (odd/even schedule)
   int *idx = nullptr, *counts = nullptr, *cu_rows = nullptr, *rowtok = nullptr, *done_ctr = nullptr;
   int* err = nullptr;
   bf16 *xn = nullptr, *q = nullptr, *o = nullptr, *hbuf = nullptr, *cacheK = nullptr,
@@ -185,6 +190,8 @@ const char* validate(const ivit_config* c) {
   if (c->ref_mode != IVIT_REF_PREV_FRAME && c->ref_mode != IVIT_REF_LAST_REFRESH) return "bad ref_mode";
   if (c->select_mode == IVIT_SEL_TOPK && c->topk < 0) return "topk must be >= 0";
   if (!std::isfinite(c->threshold)) return "threshold must be finite";
+  if (c->score_source != IVIT_SCORE_EMBED && c->score_source != IVIT_SCORE_KEY0) return "bad score_source";
+  if (c->schedule != IVIT_SCHED_INCREMENTAL && c->schedule != IVIT_SCHED_ODD_EVEN) return "bad schedule";
   return nullptr;
 }
 
@@ -447,6 +454,8 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   const size_t o_o = sa.take(M * D * 2), o_h = sa.take(M * F * 2);
   const size_t o_ck = sa.take(L * M * D * 2), o_cv = sa.take(L * M * D * 2), o_tok = sa.take(M * D * 2);
   const size_t o_err = sa.take(4);
+  const size_t o_key = c.score_source == IVIT_SCORE_KEY0 ? sa.take(M * D * 4) : 0;
+  const size_t o_rta = sa.take(M * 4), o_mall = sa.take(4);
   const size_t o_fb = sa.take(static_cast<size_t>(h->SV) * c.img_h * c.img_w * 3);
   const size_t o_cb = sa.take(h->SV * 4);
   IVIT_CK(h, cudaMalloc(&h->smem, sa.size));
@@ -470,6 +479,18 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   h->cacheV = sa.at<bf16>(o_cv);
   h->tok_out = sa.at<bf16>(o_tok);
   h->err = sa.at<int>(o_err);
+  if (c.score_source == IVIT_SCORE_KEY0) h->key_t = sa.at<float>(o_key);
+  h->rowtok_all = sa.at<int>(o_rta);
+  h->m_all = sa.at<int>(o_mall);
+  {
+    std::vector<int> ident(M);
+    for (size_t i = 0; i < M; ++i) ident[i] = static_cast<int>(i);
+    const int m_host = static_cast<int>(M);
+    IVIT_CK(h, cudaMemcpy(h->rowtok_all, ident.data(), M * sizeof(int), cudaMemcpyHostToDevice));
+    IVIT_CK(h, cudaMemcpy(h->m_all, &m_host, sizeof(int), cudaMemcpyHostToDevice));
+  }
+  if (!make_map(&h->tm_wk0, h->layers[0].wqkv + D * D, D, D, D * 2, 64, 128))
+    return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for the first-layer key projection");
   h->frames_buf = sa.at<uint8_t>(o_fb);
   h->counts_buf = sa.at<int>(o_cb);
   const int kps = ivit::attention_keys_per_split(h->N);
@@ -588,15 +609,36 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
     a.epi.ld_out = D;
     if (int r = gemm(h, plan[kGemmEmbed], h->tm_pe, h->tm_patches, a, s)) return r;
   }
+  const float* score_vec = h->e_t;
+  if (c.score_source == IVIT_SCORE_KEY0) {
+    // Eq. 3 on first-layer keys of every token: W_K LN1(e + pos) + b_K (x, xn are free
+    // until the updated rows are gathered below)
+    IVIT_CK(h, ivit::launch_gather(h->m_all, h->rowtok_all, h->e_t, h->pos, h->x, nullptr, h->e_ref, N, D, 0,
+                                   cm, M, h->row_grid, s));
+    IVIT_CK(h, ivit::launch_layernorm(h->m_all, h->x, h->layers[0].ln1g, h->layers[0].ln1b, h->xn, nullptr, D,
+                                      c.ln_eps, M, h->row_grid, s));
+    h->launches += 2;
+    ivit::GemmArgs a;
+    a.n_out = D;
+    a.k = D;
+    a.m_static = M;
+    a.epi.kind = ivit::kEpiF32Bias;
+    a.epi.bias = h->layers[0].bqkv + D;
+    a.epi.out_f32 = h->key_t;
+    a.epi.ld_out = D;
+    // a D x D projection of every row: the full encode's out-projection launch shape
+    if (int r = gemm(h, h->plan_full[kGemmO], h->tm_wk0, h->tm_xn, a, s)) return r;
+    score_vec = h->key_t;
+  }
   if (!full) {
-    IVIT_CK(h, ivit::launch_score(h->e_t, h->e_ref, h->sims, M, D, c.ref_mode == IVIT_REF_PREV_FRAME, s));
+    IVIT_CK(h, ivit::launch_score(score_vec, h->e_ref, h->sims, M, D, c.ref_mode == IVIT_REF_PREV_FRAME, s));
     ++h->launches;
   }
   IVIT_CK(h, ivit::launch_select(h->sims, N, SV, full ? IVIT_SEL_THRESHOLD : c.select_mode, c.threshold,
                                  c.topk, cm, h->idx, h->counts, h->cu_rows, h->rowtok, h->done_ctr,
                                  user_counts, s));
   ++h->launches;
-  IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, h->x, h->e_ref, N, D,
+  IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, h->x, score_vec, h->e_ref, N, D,
                                  c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
   ++h->launches;
 
@@ -712,7 +754,7 @@ int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_coun
     IVIT_CK(h, cudaMemcpyAsync(h->frames_buf, frames, fbytes, cudaMemcpyDeviceToDevice, s));
     IVIT_CK(h, cudaGraphLaunch(*exec, s));
     if (out) IVIT_CK(h, cudaMemcpyAsync(out, h->tok_out, tok_bytes, cudaMemcpyDeviceToDevice, s));
-    if (user_counts && !full)
+    if (user_counts)
       IVIT_CK(h, cudaMemcpyAsync(user_counts, h->counts_buf, SV * sizeof(int), cudaMemcpyDeviceToDevice, s));
     h->launches = *nl;
   } else {
@@ -785,7 +827,9 @@ int ivit_encode_incremental(ivit_handle* h, const uint8_t* frames_dev, uint16_t*
                             int32_t* changed_count_dev, void* stream) {
   if (!h) return IVIT_ERR_ARG;
   if (!frames_dev) return h->fail(IVIT_ERR_ARG, "null frames");
-  return run(h, frames_dev, tokens_out_dev, changed_count_dev, false, static_cast<cudaStream_t>(stream));
+  // odd/even chunks (Sec. III-B): the 1st, 3rd, ... call is a full forward
+  const bool full = h->cfg.schedule == IVIT_SCHED_ODD_EVEN && (h->chunk++ % 2) == 0;
+  return run(h, frames_dev, tokens_out_dev, changed_count_dev, full, static_cast<cudaStream_t>(stream));
 }
 
 int ivit_get_changed(ivit_handle* h, int sv, int32_t* idx_dev, int32_t* count_dev, void* stream) {

@@ -133,9 +133,11 @@ cudaError_t launch_select(const float* sims, int n_tok, int sv, int mode, float 
                           const ColdMask& cold, int* idx, int* counts, int* cu_rows, int* rowtok,
                           int* done_ctr, int* user_counts, cudaStream_t s);
 
+// x[r] = e_t[tok] + pos[tok % N] for the packed rows; refreshes e_ref[tok] from
+// ref_src[tok] for refreshed tokens (last-refresh reference or cold view).
 cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const float* e_t,
-                          const float* pos, float* x, float* e_ref, int n_tok, int dim,
-                          int ref_last_refresh, const ColdMask& cold, int max_rows, int grid,
+                          const float* pos, float* x, const float* ref_src, float* e_ref, int n_tok,
+                          int dim, int ref_last_refresh, const ColdMask& cold, int max_rows, int grid,
                           cudaStream_t s);
 
 // y[r] = LN(x[r]) (bf16) for r < *rows; when dst_rowtok is set, row r is written to

@@ -166,12 +166,14 @@ __global__ void select_kernel(const float* __restrict__ sims, int N, int sv, int
 
 // ----------------------------------------------------------------------- gather
 // x[r] = e_t[tok] + pos[tok % N] for the packed updated rows (fp32 residual stream).
-// The reference row of an updated token is refreshed here when the reference is the
-// last refresh, or when the view was cold.
+// The reference row of an updated token (e_ref[tok] <- ref_src[tok], the score vector:
+// patch embedding or first-layer key) is refreshed here when the reference is the last
+// refresh, or when the view was cold.  ref_src may be null (no refresh).
 __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __restrict__ rowtok,
                               const float* __restrict__ e_t, const float* __restrict__ pos,
-                              float* __restrict__ x, float* __restrict__ e_ref, int N, int dim,
-                              int ref_last_refresh, const ColdMask cold) {
+                              float* __restrict__ x, const float* __restrict__ ref_src,
+                              float* __restrict__ e_ref, int N, int dim, int ref_last_refresh,
+                              const ColdMask cold) {
   pdl_wait();
   pdl_launch_dependents();
   const int rows = *total_rows;
@@ -180,15 +182,18 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
   for (int r = blockIdx.x * warps + (threadIdx.x >> 5); r < rows; r += gridDim.x * warps) {
     const int tok = rowtok[r];
     const int ti = tok % N;
-    const bool refresh = ref_last_refresh || is_cold(cold, tok / N);
+    const bool refresh = ref_src && (ref_last_refresh || is_cold(cold, tok / N));
     const float4* a = reinterpret_cast<const float4*>(e_t + static_cast<size_t>(tok) * dim);
     const float4* p = reinterpret_cast<const float4*>(pos + static_cast<size_t>(ti) * dim);
     float4* y = reinterpret_cast<float4*>(x + static_cast<size_t>(r) * dim);
-    float4* er = reinterpret_cast<float4*>(e_ref + static_cast<size_t>(tok) * dim);
     for (int c = lane; c < dim / 4; c += 32) {
       const float4 u = a[c], w = p[c];
       y[c] = make_float4(u.x + w.x, u.y + w.y, u.z + w.z, u.w + w.w);
-      if (refresh) er[c] = u;
+    }
+    if (refresh) {
+      const float4* src = reinterpret_cast<const float4*>(ref_src + static_cast<size_t>(tok) * dim);
+      float4* er = reinterpret_cast<float4*>(e_ref + static_cast<size_t>(tok) * dim);
+      for (int c = lane; c < dim / 4; c += 32) er[c] = src[c];
     }
   }
 }
@@ -499,12 +504,12 @@ cudaError_t launch_select(const float* sims, int n_tok, int sv, int mode, float 
 }
 
 cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const float* e_t,
-                          const float* pos, float* x, float* e_ref, int n_tok, int dim,
-                          int ref_last_refresh, const ColdMask& cold, int max_rows, int grid,
+                          const float* pos, float* x, const float* ref_src, float* e_ref, int n_tok,
+                          int dim, int ref_last_refresh, const ColdMask& cold, int max_rows, int grid,
                           cudaStream_t s) {
   grid = max(1, min(grid, (max_rows + 7) / 8));
   return launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, 1, cu_rows_total, rowtok, e_t, pos, x,
-                   e_ref, n_tok, dim, ref_last_refresh, cold);
+                   ref_src, e_ref, n_tok, dim, ref_last_refresh, cold);
 }
 
 cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma, const float* beta,

@@ -31,15 +31,15 @@ def assert_tokens_close(gpu: np.ndarray, ref: np.ndarray, what: str = ""):
 
 def run_side_by_side(pkg, oracle_mod, shape, weights, frames, n_streams=1, n_views=1,
                      select_mode=0, threshold=0.98, topk=0, ref_mode=0, margin=2e-3,
-                     check_caches=False, first_full=True):
+                     check_caches=False, first_full=True, score_source=0, schedule=0):
     """Feeds ``frames`` (list of uint8 [SV,H,W,3]) to both sides; frame 0 is a full
     encode when ``first_full``.  Returns per-frame (rel, cos, counts)."""
     import torch
 
     enc = pkg.IncrementalViT(shape, weights, n_streams, n_views, select_mode, threshold, topk,
-                             ref_mode)
+                             ref_mode, score_source, schedule)
     orc = oracle_mod.Oracle(shape, weights, n_streams, n_views, select_mode, threshold, topk,
-                            ref_mode)
+                            ref_mode, score_source, schedule)
     sv = n_streams * n_views
     stats = []
     try:
@@ -57,6 +57,11 @@ def run_side_by_side(pkg, oracle_mod, shape, weights, frames, n_streams=1, n_vie
                 if select_mode == 0 and warm.any():
                     gap = np.abs(sims[warm] - threshold).min()
                     assert gap > margin, f"frame {t}: a score is within {gap} of the threshold"
+                if select_mode == 1 and 0 < topk < shape.n_tokens:
+                    for v in np.nonzero(warm)[0]:  # the k-th and (k+1)-th scores must separate
+                        srt = np.sort(sims[v])
+                        assert srt[topk] - srt[topk - 1] > margin, (
+                            f"frame {t} view {v}: top-{topk} boundary gap {srt[topk] - srt[topk - 1]}")
                 np.testing.assert_array_equal(counts, rc, err_msg=f"frame {t}: counts")
                 for v in range(sv):
                     np.testing.assert_array_equal(enc.changed(v).cpu().numpy(), ridx[v, :rc[v]],
@@ -72,7 +77,10 @@ def run_side_by_side(pkg, oracle_mod, shape, weights, frames, n_streams=1, n_vie
                     assert_tokens_close(g, r, f"cache {which} layer {l}")
             g = enc.cache("ref").cpu().numpy()
             r = orc.cache("ref")
-            assert np.abs(g - r).max() <= 1e-4 * np.abs(r).max() + 1e-6, "reference embeddings"
+            if score_source == 0:  # patch embeddings: exact bf16 products, fp32 sums
+                assert np.abs(g - r).max() <= 1e-4 * np.abs(r).max() + 1e-6, "reference embeddings"
+            else:  # first-layer keys: a bf16 GEMM over the bf16 LN output
+                assert_tokens_close(g, r, "reference keys")
         assert enc.device_status() == 0
     finally:
         enc.close()

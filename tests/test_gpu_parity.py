@@ -110,9 +110,11 @@ def test_reset_one_stream(pkg, oracle_mod):
 
 @pytest.mark.parametrize("k", [0, 1, 7, 64])
 def test_topk_selection(pkg, oracle_mod, k):
+    # k patches repainted per frame (7 when k selects none or all): the k lowest scores
+    # are separated from the others by a margin, so the selection is well-posed
     shape = SHAPE_A
     w = synth.make_weights(shape, 17)
-    frames = list(synth.stream_repaint(shape, 2, 3, 7, 18))
+    frames = list(synth.stream_repaint(shape, 2, 3, k if 0 < k < shape.n_tokens else 7, 18))
     stats = run_side_by_side(pkg, oracle_mod, shape, w, frames, 1, 2,
                              select_mode=synth.SEL_TOPK, topk=k)
     for s in stats[1:]:
@@ -142,3 +144,38 @@ def test_both_execution_paths(pkg, oracle_mod, forced_path, shape, S, V):
     frames = list(synth.stream_random(shape, S * V, 4, 26, change_p=0.15))
     run_side_by_side(pkg, oracle_mod, shape, w, frames, S, V, check_caches=True)
     run_side_by_side(pkg, oracle_mod, shape, w, frames[:2], S, V, first_full=False)
+
+
+@pytest.mark.parametrize("forced_path", ["kernels", "persistent"], indirect=True)
+@pytest.mark.parametrize("mode,k", [(synth.SEL_THRESHOLD, 0), (synth.SEL_TOPK, 11)])
+def test_first_layer_key_scores(pkg, oracle_mod, forced_path, mode, k):
+    # Eq. 3 as printed: cosine of the first layer's keys of every token.  Top-k repaints
+    # exactly k patches per view so the k lowest scores are well separated from the rest.
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 27)
+    if mode == synth.SEL_TOPK:
+        frames = list(synth.stream_repaint(shape, 3, 4, k, 28))
+    else:
+        frames = list(synth.stream_random(shape, 3, 4, 28, change_p=0.2))
+    run_side_by_side(pkg, oracle_mod, shape, w, frames, 1, 3, select_mode=mode, topk=k,
+                     score_source=synth.SCORE_KEY0, check_caches=True)
+
+
+def test_first_layer_key_scores_last_refresh(pkg, oracle_mod):
+    shape = SHAPE_C
+    w = synth.make_weights(shape, 29)
+    frames = list(synth.stream_random(shape, 2, 4, 30, change_p=0.3))
+    run_side_by_side(pkg, oracle_mod, shape, w, frames, 1, 2, score_source=synth.SCORE_KEY0,
+                     ref_mode=synth.REF_LAST_REFRESH, check_caches=True)
+
+
+def test_odd_even_schedule(pkg, oracle_mod):
+    # every call through ivit_encode_incremental: odd calls encode in full (count N)
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 31)
+    frames = list(synth.stream_random(shape, 2, 5, 32, change_p=0.2))
+    stats = run_side_by_side(pkg, oracle_mod, shape, w, frames, 1, 2, first_full=False,
+                             score_source=synth.SCORE_KEY0, schedule=synth.SCHED_ODD_EVEN)
+    N = shape.n_tokens
+    assert [s[2].tolist() for s in stats[0::2]] == [[N, N]] * 3
+    assert all(s[2].max() < N for s in stats[1::2])
