@@ -162,17 +162,32 @@ def cpu_baseline(wl, weights, frames, budget_s: float = 20.0) -> dict:
     orc = oracle.Oracle.for_workload(wl, weights)
     orc.encode_full(frames[0])
     done, t0 = 0, time.perf_counter()
-    while done + 1 < len(frames):
+    while done + 3 < len(frames):  # keeps two frames for the single-thread leg
         orc.encode_incremental(frames[done + 1])
         done += 1
         if time.perf_counter() - t0 > budget_s:
             break
     el = time.perf_counter() - t0
-    orc.close()
     cores = len(os.sched_getaffinity(0))
+    # the same oracle state continued on one thread (bounded to a few frames)
+    single = None
+    if done + 1 < len(frames):
+        oracle.set_threads(1)
+        n1, t1 = 0, time.perf_counter()
+        while done + 1 + n1 < len(frames):
+            orc.encode_incremental(frames[done + 1 + n1])
+            n1 += 1
+            if time.perf_counter() - t1 > budget_s / 2:
+                break
+        el1 = time.perf_counter() - t1
+        oracle.set_threads(cores)
+        single = {"value": n1 * wl.sv / el1, "unit": "frames/s", "cores": 1,
+                  "sample": f"frames {done + 1}..{done + n1} of the same stream ({el1:.1f} s)"}
+    orc.close()
     return {"value": done * wl.sv / el, "unit": "frames/s", "cores": cores, "kind": "oracle",
             "sample": (f"oracle incremental encode of frames 1..{done} of the {wl.name} stream after an "
-                       f"untimed full encode of frame 0 ({el:.1f} s, OpenMP over {cores} cores)")}
+                       f"untimed full encode of frame 0 ({el:.1f} s, OpenMP over {cores} cores)"),
+            "single_thread": single}
 
 
 def run_reference(args, wl, rank: int) -> None:
@@ -258,21 +273,27 @@ def main() -> None:
 
     host_ms = {}
 
+    step_ms = {}
+
     def timed(fn_step, label):
-        """Full encode of frame 0, warm-up frames, then K timed steps (CUDA events)."""
+        """Full encode of frame 0, warm-up frames, then K timed steps (CUDA events on the
+        launch stream, one after every step for the per-step distribution)."""
         enc.encode_full(frames_dev[0], out)
         for t in range(args.warmup):
             fn_step(1 + t)
         barrier()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+        ev[0].record(stream)
         h0 = time.perf_counter()
         for t in range(args.steps):
             fn_step(1 + args.warmup + t)
+            ev[t + 1].record(stream)
         host_ms[label] = 1e3 * (time.perf_counter() - h0) / args.steps
-        e1.record(stream)
-        e1.synchronize()
-        ms = e0.elapsed_time(e1)
+        ev[-1].synchronize()
+        ms = ev[0].elapsed_time(ev[-1])
+        per = np.array([ev[i].elapsed_time(ev[i + 1]) for i in range(args.steps)])
+        step_ms[label] = {"median": float(np.median(per)), "p10": float(np.percentile(per, 10)),
+                          "p90": float(np.percentile(per, 90))}
         barrier()
         return max_over_ranks(ms, dist, dev)
 
@@ -331,6 +352,8 @@ def main() -> None:
             "dynamic_fraction_mean": float(changed.mean()) / (wl.sv * wl.shape.n_tokens),
         }),
         "ms_per_frame": inc_ms / args.steps / wl.sv,
+        "timesteps_per_s": args.steps * world / (inc_ms / 1e3),
+        "ms_per_step_distribution": step_ms,
         "full_encode_ms_per_step": full_ms / args.steps,
         "full_encode_frames_per_s": frames_total / (full_ms / 1e3),
         "speedup_vs_full": full_ms / inc_ms,
