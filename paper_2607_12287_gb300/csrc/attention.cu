@@ -1,0 +1,485 @@
+// Attention of the updated queries of every view over all N keys of that view, on the
+// tensor cores (Sec. III-B: attention is computed only for the updated tokens; Eq. 5:
+// the keys and values of reused tokens come from the per-layer cache):
+//
+//   O = softmax(Q K^T / sqrt(dh)) V          per (view, head).
+//
+// Work item = (query tile of up to 128 packed updated rows of view v, head h).  Each
+// item is handled by a thread-block cluster of `ns` CTAs that split the view's keys:
+// CTA rank s takes keys [s*kpc, (s+1)*kpc), kpc = ceil(N / ns) <= 256.  The clusters
+// walk the items with a stride; items past a view's row count (device-resident, written
+// by the selection kernel) are skipped, so one launch shape serves every row count and
+// the launch can sit in a CUDA graph.  Shared memory and TMEM are sized by kpc, so that
+// with 64 keys per CTA an attention CTA fits on an SM beside a GEMM CTA and starts (and
+// prefetches) while the QKV GEMM is still running.
+//
+// Per item and CTA, 128 threads; thread i <-> query row i <-> TMEM lane i:
+//   Q tile [128 rows][dh] by TMA (128-byte swizzle, 64-column slices; the padding columns
+//   dh..round16(dh) are zeroed in shared memory); K, V of the CTA's keys by TMA into
+//   [kpc keys][64 columns] slices;
+//   S = Q K^T   tcgen05.mma M = 128, N = the CTA's keys, K = round16(dh), fp32 in TMEM;
+//   softmax     each thread reads its row of S from TMEM; row max m, P = 2^((S - m) c)
+//               (c = log2(e) / sqrt(dh)) rounded to bf16 into shared memory as the next
+//               MMA's A operand (K-major, 128-byte swizzle), l = the sum of those values;
+//   O_s = P V   V is the B operand in MN-major form (its rows are the keys = the MMA's
+//               K, its columns the head's dims = the MMA's N): one MMA for dims 0..63
+//               and one for the rest, each inside one 64-column swizzle atom;
+//   merge       every CTA stores the partial (m, l, O_s) of each row into the shared
+//               memory of the row's owner CTA (distributed shared memory stores); after
+//               a cluster barrier the owner combines them in rank order (deterministic):
+//               M = max m_s,  O = sum_s 2^((m_s - M) c) O_s / sum_s 2^((m_s - M) c) l_s.
+// Incremental calls fetch the cached K/V of the item's view before waiting on the QKV
+// kernel (programmatic dependent launch: reused tokens' keys are final) and afterwards
+// copy only the rows of this call's updated tokens into the swizzled tiles.
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace ivit {
+namespace {
+
+constexpr int AQ = 128;            // queries per item (MMA M)
+constexpr int AKMAX = 256;         // max keys per CTA (MMA N of S)
+constexpr int KROWS = 64;          // rows of one K/V TMA box
+constexpr int SLICE_Q = AQ * 128;  // [128 rows][128 B]: 16 KB (a Q slice or a 64-key P slice)
+constexpr int MAX_SPLITS = 8;
+
+// Shared-memory and TMEM layout of one CTA for kpc keys and head width dhp (padded to
+// 16), identical on host and device.
+struct AttnLayout {
+  int nsl;       // 64-column slices per row
+  int kpad;      // keys per CTA rounded up to 64 (K/V slice rows)
+  int kslice;    // bytes of one K or V slice
+  int rp, pst;   // merge: row slots per owner, row stride of a partial output (floats)
+  int off_q, off_p, off_k, off_v, off_part, off_bar, bytes;
+  int tm_o, tm_cols;
+};
+
+__host__ __device__ inline AttnLayout attn_layout(int kpc, int dhp, int ns) {
+  AttnLayout L;
+  L.nsl = dhp > 64 ? 2 : 1;
+  L.kpad = (kpc + 63) / 64 * 64;
+  L.kslice = L.kpad * 128;
+  L.rp = (AQ + ns - 1) / ns;
+  L.pst = dhp + 4;
+  L.off_q = 0;
+  L.off_p = L.off_q + L.nsl * SLICE_Q;
+  L.off_k = L.off_p + (L.kpad / 64) * SLICE_Q;
+  L.off_v = L.off_k + L.nsl * L.kslice;
+  L.off_part = L.off_v + L.nsl * L.kslice;
+  const int part = ns > 1 ? ns * L.rp * (L.pst + 2) * 4 : 0;  // O_s, m, l of every slot
+  L.off_bar = L.off_part + (part + 1023) / 1024 * 1024;
+  L.bytes = L.off_bar + 64 + 1024;  // barriers + TMEM slot, alignment slack
+  L.tm_o = L.kpad;
+  int need = L.kpad + dhp, cols = 32;
+  while (cols < need) cols *= 2;
+  L.tm_cols = cols;
+  return L;
+}
+
+// Byte offset of 16-byte chunk `chunk` (0..7) of row `row` in a slice of 128-byte rows
+// written by TMA with 128-byte swizzle (slice base 1024-byte aligned).
+__device__ __forceinline__ uint32_t swz(int row, int chunk) {
+  return static_cast<uint32_t>(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
+struct Item {
+  int v, h, r0, nq;
+};
+
+// Item s = (query tile, view, head) with the query tile slowest, so that the first
+// tiles of every (view, head) are spread over the grid first.
+__device__ __forceinline__ bool item_at(int s, const AttnTcArgs& a, Item& it) {
+  const int vh = a.sv * a.heads;
+  const int qt = s / vh, rem = s - qt * vh;
+  it.v = rem / a.heads;
+  it.h = rem - it.v * a.heads;
+  const int rb = a.cu_rows[it.v], m = a.cu_rows[it.v + 1] - rb;
+  it.r0 = rb + qt * AQ;
+  it.nq = min(AQ, m - qt * AQ);
+  return it.nq > 0;
+}
+
+// 2^x (the softmax's exponentials on logits pre-scaled by log2(e) / sqrt(dh)).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+template <int DHP>
+__global__ void __launch_bounds__(128, 1)
+    attention_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                        const __grid_constant__ CUtensorMap tm_v, const AttnTcArgs a) {
+  extern __shared__ uint8_t at_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(at_raw) + 1023) &
+                                           ~static_cast<uintptr_t>(1023));
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int N = a.n_tok, D = a.dim, dh = a.dh;
+  const int n_items = a.sv * a.heads * a.qtiles;
+  const int ns = static_cast<int>(cluster_nctarank()), rank = static_cast<int>(cluster_ctarank());
+  const int cl = blockIdx.x / ns, ncl = gridDim.x / ns;
+  const int kpc = (N + ns - 1) / ns;
+  const int k0 = rank * kpc, nk = max(0, min(kpc, N - k0)), nks = (nk + 15) & ~15;
+  const AttnLayout L = attn_layout(kpc, DHP, ns);
+  const int NSL = L.nsl;
+  const uint32_t sb = smem_u32(sm);
+  const uint32_t bq = sb + L.off_bar, bk = bq + 8, bv = bq + 16, bs = bq + 24, bo = bq + 32;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + L.off_bar + 40);
+  // merge slots of the rows this CTA owns: O_s [ns][rp][pst], then m [ns][rp], l [ns][rp]
+  float* po = reinterpret_cast<float*>(sm + L.off_part);
+  float* pm = po + ns * L.rp * L.pst;
+  float* pl = pm + ns * L.rp;
+
+  // The row offsets come from the selection kernel, at least two launches back (every
+  // kernel of the library triggers its dependents only after its own wait).  Every CTA
+  // of a cluster walks the same items, so a cluster leaves as a whole.
+  int s = cl;
+  Item it;
+  while (s < n_items && !item_at(s, a, it)) s += ncl;
+  if (s >= n_items) return;
+
+  if (tid == 0) {
+    mbar_init(bq, 1);
+    mbar_init(bk, 1);
+    mbar_init(bv, 1);
+    mbar_init(bs, 1);
+    mbar_init(bo, 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_k);
+    tma_prefetch_desc(&tm_v);
+  }
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tslot), static_cast<uint32_t>(L.tm_cols));
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+  const uint32_t tm_s = tmem, tm_o = tmem + static_cast<uint32_t>(L.tm_o);
+  const uint64_t pol_q = l2_policy_evict_first(), pol_kv = l2_policy_evict_last();
+
+  // K or V of this CTA's keys of item (v, h): boxes of 64 keys x 64 dims per slice.
+  auto load_kv = [&](uint32_t bar, int off, const CUtensorMap* map, int v, int h) {
+    const int nbox = (nk + KROWS - 1) / KROWS;
+    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(nbox * NSL * KROWS * 128));
+    for (int sl = 0; sl < NSL; ++sl)
+      for (int b = 0; b < nbox; ++b)
+        tma_load_2d(sb + off + sl * L.kslice + b * KROWS * 128, map, h * dh + sl * 64, v * N + k0 + b * KROWS,
+                    bar, pol_kv);
+  };
+
+  if (a.prefetch && tid == 0) {
+    load_kv(bk, L.off_k, &tm_k, it.v, it.h);
+    load_kv(bv, L.off_v, &tm_v, it.v, it.h);
+  }
+  pdl_wait();  // queries and this call's K/V rows (QKV kernel) are visible from here
+  pdl_launch_dependents();
+
+  uint32_t ph = 0;  // completed phases of every barrier (each completes once per item)
+  bool ok = true;
+  const float sc = rsqrtf(static_cast<float>(dh)) * 1.4426950408889634f;  // log2(e) / sqrt(dh)
+  bool first = true;
+  while (true) {
+    const bool patch = first && a.prefetch;
+    first = false;
+    if (tid == 0) {
+      mbar_arrive_expect_tx(bq, NSL * SLICE_Q);
+      for (int sl = 0; sl < NSL; ++sl)
+        tma_load_2d(sb + L.off_q + sl * SLICE_Q, &tm_q, it.h * dh + sl * 64, it.r0, bq, pol_q);
+      if (!patch) {
+        load_kv(bk, L.off_k, &tm_k, it.v, it.h);
+        load_kv(bv, L.off_v, &tm_v, it.v, it.h);
+      }
+    }
+    if (patch) {
+      // the prefetched tiles hold the cache as it was before the QKV kernel: overwrite
+      // the rows of the tokens it updated that fall in this CTA's key range
+      if (!mbar_wait(bk, ph & 1) || !mbar_wait(bv, ph & 1)) ok = false;
+      const int rb = a.cu_rows[it.v], m = a.cu_rows[it.v + 1] - rb;
+      const int dh8 = dh >> 3;
+      for (int e = tid; e < m * dh8; e += blockDim.x) {
+        const int r = e / dh8, c = e - r * dh8;
+        const int j = a.rowtok[rb + r] - it.v * N - k0;
+        if (j < 0 || j >= nk) continue;
+        const size_t g = (static_cast<size_t>(it.v) * N + k0 + j) * D + it.h * dh + c * 8;
+        const uint32_t off = (c >> 3) * L.kslice + swz(j, c & 7);
+        *reinterpret_cast<uint4*>(sm + L.off_k + off) = __ldcg(reinterpret_cast<const uint4*>(a.cache_k + g));
+        *reinterpret_cast<uint4*>(sm + L.off_v + off) = __ldcg(reinterpret_cast<const uint4*>(a.cache_v + g));
+      }
+    }
+    if (!mbar_wait(bq, ph & 1)) ok = false;
+    if (DHP != dh) {  // columns dh..dh+7 of the Q tile hold the next head: zero them
+      const int c = dh >> 3;
+      *reinterpret_cast<uint4*>(sm + L.off_q + (c >> 3) * SLICE_Q + swz(tid, c & 7)) = make_uint4(0, 0, 0, 0);
+    }
+    fence_proxy_async_shared();
+    tc_fence_before();
+    __syncthreads();
+
+    // ---- S = Q K^T
+    if (tid == 0) {
+      tc_fence_after();
+      if (!mbar_wait(bk, ph & 1)) ok = false;
+      tc_fence_after();
+      if (ok && nk > 0) {
+        const uint32_t id = idesc_bf16_f32(AQ, nks);
+#pragma unroll
+        for (int t = 0; t < DHP / 16; ++t) {
+          const uint32_t qo = sb + L.off_q + (t >> 2) * SLICE_Q + (t & 3) * 32;
+          const uint32_t ko = sb + L.off_k + (t >> 2) * L.kslice + (t & 3) * 32;
+          umma_bf16(tm_s, sdesc_kmajor_sw128(qo), sdesc_kmajor_sw128(ko), id, t > 0);
+        }
+      }
+      umma_commit(bs);
+    }
+    __syncwarp();
+    if (!mbar_wait(bs, ph & 1)) ok = false;
+    tc_fence_after();
+
+    // ---- softmax over this CTA's keys, P to shared memory
+    const bool wact = warp * 32 < it.nq && nk > 0;  // warp-uniform; padding warps skip the math
+    float m_run = -INFINITY, l_run = 0.f;
+    if (wact) {
+      for (int cb = 0; cb < nks; cb += 64) {
+        uint32_t r0[32], r1[32];
+        tmem_ld32_async(trow + cb, r0);
+        tmem_ld32_async(trow + cb + 32, r1);
+        tmem_ld_wait();
+#pragma unroll
+        for (int u = 0; u < 32; ++u) {
+          if (cb + u < nk) m_run = fmaxf(m_run, __uint_as_float(r0[u]));
+          if (cb + 32 + u < nk) m_run = fmaxf(m_run, __uint_as_float(r1[u]));
+        }
+      }
+      const float mo = m_run * sc;
+      float lsum[4] = {0.f, 0.f, 0.f, 0.f};
+      for (int cb = 0; cb < nks; cb += 32) {
+        uint32_t r[32];
+        tmem_ld32_async(trow + cb, r);
+        tmem_ld_wait();
+        uint32_t pk[16];
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const int j = cb + 2 * u;
+          const float p0 = j < nk ? ex2(fmaf(__uint_as_float(r[2 * u]), sc, -mo)) : 0.f;
+          const float p1 = j + 1 < nk ? ex2(fmaf(__uint_as_float(r[2 * u + 1]), sc, -mo)) : 0.f;
+          const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
+          const float2 f = __bfloat1622float2(b);
+          lsum[u & 3] += f.x + f.y;  // the normaliser sums the values the MMA multiplies
+          pk[u] = *reinterpret_cast<const uint32_t*>(&b);
+        }
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+          const int kc = (cb >> 3) + q4;  // 16-byte chunk (8 keys) of this row of P
+          if (kc * 8 < nks)
+            *reinterpret_cast<uint4*>(sm + L.off_p + (kc >> 3) * SLICE_Q + swz(tid, kc & 7)) =
+                make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
+        }
+      }
+      l_run = (lsum[0] + lsum[1]) + (lsum[2] + lsum[3]);
+    }
+    fence_proxy_async_shared();
+    tc_fence_before();
+    __syncthreads();
+
+    // ---- O_s = P V
+    if (tid == 0) {
+      tc_fence_after();
+      if (!mbar_wait(bv, ph & 1)) ok = false;
+      tc_fence_after();
+      if (ok && nk > 0) {
+        const uint32_t id0 = idesc_bf16_f32_bmn(AQ, DHP > 64 ? 64 : DHP);
+        const uint32_t id1 = idesc_bf16_f32_bmn(AQ, DHP > 64 ? DHP - 64 : 16);
+        for (int t = 0; t < nks / 16; ++t) {
+          const uint64_t ad = sdesc_kmajor_sw128(sb + L.off_p + (t >> 2) * SLICE_Q + (t & 3) * 32);
+          umma_bf16(tm_o, ad, sdesc_sw128(sb + L.off_v + t * 2048, 1024, 1024), id0, t > 0);
+          if (DHP > 64)
+            umma_bf16(tm_o + 64, ad, sdesc_sw128(sb + L.off_v + L.kslice + t * 2048, 1024, 1024), id1, t > 0);
+        }
+      }
+      umma_commit(bo);
+    }
+    __syncwarp();
+    if (!mbar_wait(bo, ph & 1)) ok = false;
+    tc_fence_after();
+    ++ph;
+
+    // next item of this cluster (the same for every rank)
+    int s_next = s + ncl;
+    Item nxt;
+    while (s_next < n_items && !item_at(s_next, a, nxt)) s_next += ncl;
+
+    if (ns == 1) {
+      if (wact) {  // warp-uniform: tcgen05.ld is a warp-collective instruction
+        const float inv = 1.f / l_run;
+        bf16* orow = a.o + static_cast<size_t>(it.r0 + tid) * D + it.h * dh;
+#pragma unroll
+        for (int c = 0; c < DHP; c += 16) {
+          float ov[16];
+          tmem_ld16(trow + L.tm_o + c, ov);
+#pragma unroll
+          for (int h8 = 0; h8 < 16; h8 += 8) {
+            if (tid < it.nq && c + h8 < dh) {
+              uint4 u;
+              uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const __nv_bfloat162 b =
+                    __floats2bfloat162_rn(ov[h8 + 2 * e] * inv, ov[h8 + 2 * e + 1] * inv);
+                w[e] = *reinterpret_cast<const uint32_t*>(&b);
+              }
+              *reinterpret_cast<uint4*>(orow + c + h8) = u;
+            }
+          }
+        }
+      }
+    } else {
+      // push this CTA's partial (m, l, O_s) of row i to slot [rank][i - owner * rpi] of
+      // the owner CTA i / rpi; key-less CTAs push a neutral partial (m = -inf, l = 0)
+      const int rpi = (it.nq + ns - 1) / ns;  // rows per owner in this item (<= rp)
+      const bool mine = tid < it.nq;
+      const int owner = mine ? tid / rpi : 0, slot = tid - owner * rpi;
+      const uint32_t obase = mapa_shared(smem_u32(po + (rank * L.rp + slot) * L.pst), static_cast<uint32_t>(owner));
+      if (warp * 32 < it.nq) {  // warp-uniform
+        if (wact) {
+#pragma unroll
+          for (int c = 0; c < DHP; c += 16) {
+            float ov[16];
+            tmem_ld16(trow + L.tm_o + c, ov);
+            if (mine)
+#pragma unroll
+              for (int q = 0; q < 16; q += 4)
+                st_dsmem_f32x4(obase + 4 * (c + q), make_float4(ov[q], ov[q + 1], ov[q + 2], ov[q + 3]));
+          }
+        } else if (mine) {
+#pragma unroll
+          for (int c = 0; c < DHP; c += 4) st_dsmem_f32x4(obase + 4 * c, make_float4(0.f, 0.f, 0.f, 0.f));
+        }
+        if (mine) {
+          st_dsmem_f32(mapa_shared(smem_u32(pm + rank * L.rp + slot), static_cast<uint32_t>(owner)), m_run);
+          st_dsmem_f32(mapa_shared(smem_u32(pl + rank * L.rp + slot), static_cast<uint32_t>(owner)), l_run);
+        }
+      }
+      cluster_sync();  // every rank's partials of this CTA's rows are in its shared memory
+      const int lo = rank * rpi, nmine = max(0, min(it.nq, lo + rpi) - lo);
+      constexpr int C8 = DHP / 8;
+      for (int e = tid; e < nmine * C8; e += blockDim.x) {
+        const int sl = e / C8, c = e - sl * C8;
+        if (c * 8 >= dh) continue;
+        float M = -INFINITY;
+#pragma unroll
+        for (int q = 0; q < MAX_SPLITS; ++q)
+          if (q < ns) M = fmaxf(M, pm[q * L.rp + sl]);
+        float Lsum = 0.f, acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int q = 0; q < MAX_SPLITS; ++q) {
+          if (q < ns) {
+            const float w = ex2((pm[q * L.rp + sl] - M) * sc);  // m = -inf (no keys): w = 0
+            Lsum += w * pl[q * L.rp + sl];
+            const float4 x0 = *reinterpret_cast<const float4*>(po + (q * L.rp + sl) * L.pst + c * 8);
+            const float4 x1 = *reinterpret_cast<const float4*>(po + (q * L.rp + sl) * L.pst + c * 8 + 4);
+            acc[0] += w * x0.x;
+            acc[1] += w * x0.y;
+            acc[2] += w * x0.z;
+            acc[3] += w * x0.w;
+            acc[4] += w * x1.x;
+            acc[5] += w * x1.y;
+            acc[6] += w * x1.z;
+            acc[7] += w * x1.w;
+          }
+        }
+        const float inv = 1.f / Lsum;
+        uint4 u;
+        uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const __nv_bfloat162 b = __floats2bfloat162_rn(acc[2 * q] * inv, acc[2 * q + 1] * inv);
+          w[q] = *reinterpret_cast<const uint32_t*>(&b);
+        }
+        *reinterpret_cast<uint4*>(a.o + static_cast<size_t>(it.r0 + lo + sl) * D + it.h * dh + c * 8) = u;
+      }
+      if (s_next < n_items) cluster_sync();  // slots are read before the next item's pushes
+    }
+    tc_fence_before();
+    __syncthreads();  // Q, P and TMEM are reused by the next item
+
+    if (s_next >= n_items) break;
+    s = s_next;
+    it = nxt;
+  }
+
+  if (!ok) atomicExch(a.err, kErrWaitTmaFull);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 0) tmem_dealloc(tmem, static_cast<uint32_t>(L.tm_cols));
+}
+
+template <int DHP>
+cudaError_t launch_dhp(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
+                       const AttnTcArgs& a, int grid, int smem, cudaStream_t s) {
+  return launch_ex(attention_tc_kernel<DHP>, dim3(grid), dim3(128), static_cast<size_t>(smem), s,
+                   static_cast<unsigned>(a.key_splits), tm_q, tm_k, tm_v, a);
+}
+
+// The device's opt-in limit of dynamic shared memory per block (0 when unknown).
+int smem_optin() {
+  int dev = 0, v = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) return 0;
+  return v;
+}
+
+}  // namespace
+
+int attention_tc_kv_box_rows() { return KROWS; }
+
+size_t attention_tc_smem(int n_tok, int dh, int key_splits) {
+  const int kpc = (n_tok + key_splits - 1) / key_splits;
+  return static_cast<size_t>(attn_layout(kpc, (dh + 15) & ~15, key_splits).bytes);
+}
+
+cudaError_t attention_tc_setup() {
+  const int max_bytes = smem_optin();
+  if (max_bytes <= 0) return cudaErrorInvalidDevice;
+  cudaError_t e = cudaSuccess;
+  auto set = [&](auto kern) {
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, max_bytes);
+  };
+  set(attention_tc_kernel<16>);
+  set(attention_tc_kernel<32>);
+  set(attention_tc_kernel<48>);
+  set(attention_tc_kernel<64>);
+  set(attention_tc_kernel<80>);
+  set(attention_tc_kernel<96>);
+  set(attention_tc_kernel<112>);
+  set(attention_tc_kernel<128>);
+  return e;
+}
+
+cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
+                                const AttnTcArgs& a, int max_ctas, cudaStream_t s) {
+  const int ns = a.key_splits;
+  if (ns < 1 || ns > MAX_SPLITS || (a.n_tok + ns - 1) / ns > AKMAX) return cudaErrorInvalidValue;
+  const int items = a.sv * a.heads * a.qtiles;
+  const int clusters = max(1, min(items, max_ctas / ns));
+  const int grid = clusters * ns;
+  const int smem = static_cast<int>(attention_tc_smem(a.n_tok, a.dh, ns));
+  if (smem > smem_optin()) return cudaErrorInvalidValue;
+  switch ((a.dh + 15) & ~15) {
+    case 16: return launch_dhp<16>(tm_q, tm_k, tm_v, a, grid, smem, s);
+    case 32: return launch_dhp<32>(tm_q, tm_k, tm_v, a, grid, smem, s);
+    case 48: return launch_dhp<48>(tm_q, tm_k, tm_v, a, grid, smem, s);
+    case 64: return launch_dhp<64>(tm_q, tm_k, tm_v, a, grid, smem, s);
+    case 80: return launch_dhp<80>(tm_q, tm_k, tm_v, a, grid, smem, s);
+    case 96: return launch_dhp<96>(tm_q, tm_k, tm_v, a, grid, smem, s);
+    case 112: return launch_dhp<112>(tm_q, tm_k, tm_v, a, grid, smem, s);
+    case 128: return launch_dhp<128>(tm_q, tm_k, tm_v, a, grid, smem, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace ivit

@@ -26,7 +26,8 @@ struct LayerW {
   bf16 *wqkv, *wo, *w1, *w2;
   float *bqkv, *bo, *b1, *b2, *ln1g, *ln1b, *ln2g, *ln2b;
   CUtensorMap tm_qkv, tm_o, tm_1, tm_2;
-  CUtensorMap tm_ck, tm_cv;  // this layer's key / value cache, attention key-split tiles
+  CUtensorMap tm_ck, tm_cv;  // this layer's key / value cache, SIMT attention key-split tiles
+  CUtensorMap tm_ak, tm_av;  // the same caches, 64 x 128 boxes, 128-byte swizzle (tcgen05)
 };
 
 struct EventPair {
@@ -111,6 +112,9 @@ struct ivit_handle {
   float *b_pe = nullptr, *pos = nullptr, *lnfg = nullptr, *lnfb = nullptr;
   std::vector<LayerW> layers;
   CUtensorMap tm_pe, tm_patches, tm_xn, tm_o, tm_h;
+  CUtensorMap tm_qa;     // packed queries, 64 x 128 boxes, 128-byte swizzle (tcgen05 attention)
+  bool attn_tc = true;   // tensor-core attention (IVIT_ATTN=simt selects the SIMT kernel)
+  int attn_splits_full = 1, attn_splits_inc = 1;  // key splits (CTAs per item) of that kernel
 
   bf16* patches = nullptr;
   float *e_t = nullptr, *e_ref = nullptr, *sims = nullptr, *x = nullptr;
@@ -337,6 +341,30 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   IVIT_CK(h, ivit::gemm_setup(64));
   IVIT_CK(h, ivit::gemm_setup(256));
   IVIT_CK(h, ivit::attention_setup());
+  IVIT_CK(h, ivit::attention_tc_setup());
+  if (const char* at = std::getenv("IVIT_ATTN")) h->attn_tc = std::string(at) != "simt";
+  {
+    // Key splits of the tensor-core attention: at most 128 keys per CTA (when 8 splits
+    // allow it), at least 64; within that, as many as fill the SMs once for the expected
+    // items (query tiles x heads x views: all tokens when full, a tenth when incremental),
+    // then more while one CTA's shared memory exceeds the device limit.
+    int optin = 0;
+    IVIT_CK(h, cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device));
+    const int dh = h->D / h->H;
+    auto splits = [&](int m_exp) {
+      const int ns_min = std::min(8, std::max((h->N + 255) / 256, (h->N + 127) / 128));
+      const int ns_cap = std::max(ns_min, std::min(8, (h->N + 63) / 64));
+      const int items = h->SV * h->H * ((m_exp + 127) / 128);
+      int ns = std::max(ns_min, std::min(ns_cap, h->num_sms / std::max(1, items)));
+      while (ns < 8 && ivit::attention_tc_smem(h->N, dh, ns) > static_cast<size_t>(optin)) ++ns;
+      return ns;
+    };
+    h->attn_splits_full = splits(h->N);
+    h->attn_splits_inc = splits(std::max(1, h->N / 10));
+    if (ivit::attention_tc_smem(h->N, dh, h->attn_splits_full) > static_cast<size_t>(optin) ||
+        ivit::attention_tc_smem(h->N, dh, h->attn_splits_inc) > static_cast<size_t>(optin))
+      h->attn_tc = false;  // not reachable for N <= 1024, dh <= 128
+  }
   if (std::getenv("IVIT_NO_PDL")) ivit::g_use_pdl = false;
   if (std::getenv("IVIT_NO_GRAPH")) h->use_graphs = false;
   IVIT_CK(h, cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking));
@@ -497,12 +525,15 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   for (size_t l = 0; l < L; ++l) {
     const size_t off = l * M * D;
     if (!make_map(&h->layers[l].tm_ck, h->cacheK + off, D, M, D * 2, D / h->H, kps, false) ||
-        !make_map(&h->layers[l].tm_cv, h->cacheV + off, D, M, D * 2, D / h->H, kps, false))
+        !make_map(&h->layers[l].tm_cv, h->cacheV + off, D, M, D * 2, D / h->H, kps, false) ||
+        !make_map(&h->layers[l].tm_ak, h->cacheK + off, D, M, D * 2, 64, ivit::attention_tc_kv_box_rows()) ||
+        !make_map(&h->layers[l].tm_av, h->cacheV + off, D, M, D * 2, 64, ivit::attention_tc_kv_box_rows()))
       return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for a cache tile");
   }
   if (!make_map(&h->tm_patches, h->patches, h->KPAD, M, h->KPAD * 2, 64, 32) ||
       !make_map(&h->tm_xn, h->xn, D, M, D * 2, 64, 32) ||
       !make_map(&h->tm_o, h->o, D, M, D * 2, 64, 32) ||
+      !make_map(&h->tm_qa, h->q, D, M, D * 2, 64, 128) ||
       !make_map(&h->tm_h, h->hbuf, F, M, F * 2, 64, 32))
     return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
   if (int r = setup_persistent(h)) return r;
@@ -675,8 +706,27 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
       a.epi.dim = D;
       if (int r = gemm(h, plan[kGemmQKV], w.tm_qkv, h->tm_xn, a, s)) return r;
     }
-    IVIT_CK(h, ivit::launch_attention(w.tm_ck, w.tm_cv, h->q, ck, cv, h->cu_rows, h->rowtok, h->o, SV, N, D, h->H,
-                                      full ? (N + 31) / 32 : std::max(1, (N / 10 + 31) / 32), s));
+    if (h->attn_tc) {
+      ivit::AttnTcArgs at;
+      at.cache_k = ck;
+      at.cache_v = cv;
+      at.cu_rows = h->cu_rows;
+      at.rowtok = h->rowtok;
+      at.o = h->o;
+      at.err = h->err;
+      at.n_tok = N;
+      at.dim = D;
+      at.dh = D / h->H;
+      at.heads = h->H;
+      at.sv = SV;
+      at.qtiles = (N + 127) / 128;
+      at.prefetch = full ? 0 : 1;
+      at.key_splits = full ? h->attn_splits_full : h->attn_splits_inc;
+      IVIT_CK(h, ivit::launch_attention_tc(h->tm_qa, w.tm_ak, w.tm_av, at, h->num_sms, s));
+    } else {
+      IVIT_CK(h, ivit::launch_attention(w.tm_ck, w.tm_cv, h->q, ck, cv, h->cu_rows, h->rowtok, h->o, SV, N, D,
+                                        h->H, full ? (N + 31) / 32 : std::max(1, (N / 10 + 31) / 32), s));
+    }
     ++h->launches;
     {
       ivit::GemmArgs a;

@@ -163,4 +163,39 @@ cudaError_t launch_attention(const CUtensorMap& tm_k, const CUtensorMap& tm_v, c
                              const int* rowtok, bf16* o, int sv, int n_tok, int dim, int heads,
                              int query_blocks, cudaStream_t s);
 
+// ----------------------------------------------------------- attention (tcgen05)
+struct AttnTcArgs {
+  const bf16* cache_k = nullptr;  // this layer's key cache, bf16 [SV*N][D] (token-major)
+  const bf16* cache_v = nullptr;  // this layer's value cache, same layout
+  const int* cu_rows = nullptr;   // [SV+1] packed-row offsets of the views' updated rows
+  const int* rowtok = nullptr;    // packed row -> token v*N + i
+  bf16* o = nullptr;              // [rows][D] attention output, packed rows
+  int* err = nullptr;             // device error word
+  int n_tok = 0, dim = 0, dh = 0, heads = 0, sv = 0;
+  int qtiles = 0;                 // query tiles of 128 rows per (view, head): ceil(N / 128)
+  int key_splits = 1;             // CTAs per cluster splitting the keys (1..8, N/splits <= 256)
+  int prefetch = 0;               // 1: cached K/V loaded before the wait, then the updated
+                                  //    rows re-read (incremental calls)
+};
+
+// One-time function attributes of the tensor-core attention kernel.
+cudaError_t attention_tc_setup();
+
+// Rows of the K/V TMA box the tensor-core attention kernel expects (the tensor maps of
+// the caches use box 64 columns x this many rows).
+int attention_tc_kv_box_rows();
+
+// Dynamic shared memory of one tensor-core attention CTA for N keys split key_splits ways.
+size_t attention_tc_smem(int n_tok, int dh, int key_splits);
+
+// O[r] = softmax(Q[r] K_v^T / sqrt(dh)) V_v per head on the tensor cores, for the packed
+// query rows r of each view v, over the N cached keys/values of that view.  tm_q: the
+// packed queries bf16 [rows][D] with box 64 columns x 128 rows; tm_k / tm_v: this
+// layer's caches bf16 [SV*N][D] with box 64 columns x attention_tc_kv_box_rows(); all
+// three with 128-byte swizzle.  Grid: clusters of
+// key_splits CTAs (128 threads each), at most max_ctas CTAs, walking the (query tile,
+// view, head) items.
+cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
+                                const AttnTcArgs& a, int max_ctas, cudaStream_t s);
+
 }  // namespace ivit
