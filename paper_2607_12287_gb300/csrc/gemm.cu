@@ -28,6 +28,7 @@ constexpr int BM = 128;          // output features per tile (MMA M)
 constexpr int BK = 64;           // K per stage: 128-byte rows, 128-byte swizzle
 constexpr int XBOX = 32;         // rows per TMA box of the activation operand
 constexpr int STAGES = 4;
+constexpr int MAX_CLUSTER = 16;  // CTAs per cluster (non-portable size, opted in)
 constexpr int W_TILE_BYTES = BM * BK * 2;
 constexpr int XBOX_BYTES = XBOX * BK * 2;
 
@@ -236,6 +237,9 @@ __global__ void __launch_bounds__(128, 1)
         }
       }
     } else {
+      // Partials stay in each CTA's shared memory; every CTA sums a slice of the tile's
+      // rows over all CTAs through distributed shared memory (all loads of a row issued
+      // before the sum), in rank order.
       if (ok) {
         if (has_k) {
           for (int c0 = 0; c0 < rows; c0 += 16) {
@@ -251,20 +255,24 @@ __global__ void __launch_bounds__(128, 1)
       }
       cluster_sync();  // every partial of this tile is in its CTA's shared memory
       if (ok) {
-        // this CTA's slice of the tile's rows; lane owns 4 consecutive features
         const int c_lo = crank * rows / csize, c_hi = (crank + 1) * rows / csize;
         const int f4 = ft * BM + 4 * lane;
         const uint32_t part_addr = smem_u32(part);
         for (int c = c_lo + warp; c < c_hi; c += 4) {
           const uint32_t off = part_addr + static_cast<uint32_t>((c * BM + 4 * lane) * 4);
+          float4 p[MAX_CLUSTER];
+#pragma unroll
+          for (int s = 0; s < MAX_CLUSTER; ++s)
+            if (s < csize) p[s] = ld_dsmem_f32x4(mapa_shared(off, s));
           float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-          for (int s = 0; s < csize; ++s) {
-            const float4 p = ld_dsmem_f32x4(mapa_shared(off, s));
-            acc.x += p.x;
-            acc.y += p.y;
-            acc.z += p.z;
-            acc.w += p.w;
-          }
+#pragma unroll
+          for (int s = 0; s < MAX_CLUSTER; ++s)
+            if (s < csize) {
+              acc.x += p[s].x;
+              acc.y += p[s].y;
+              acc.z += p[s].z;
+              acc.w += p[s].w;
+            }
           const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
 #pragma unroll
           for (int j = 0; j < 4; ++j)
