@@ -21,6 +21,7 @@ _LIB = os.path.join(_HERE, "_build", "liboracle.so")
 GELU_TANH, GELU_ERF = 0, 1
 SCORE_EMBED, SCORE_KEY0 = 0, 1
 SCHED_INCREMENTAL, SCHED_ODD_EVEN = 0, 1
+MLP_UPDATED, MLP_ALL = 0, 1
 SEL_THRESHOLD, SEL_TOPK = 0, 1
 REF_PREV_FRAME, REF_LAST_REFRESH = 0, 1
 
@@ -32,7 +33,7 @@ class OrcConfig(C.Structure):
         ("mlp_dim", C.c_int32), ("n_streams", C.c_int32), ("n_views", C.c_int32),
         ("ln_eps", C.c_float), ("gelu", C.c_int32), ("select_mode", C.c_int32),
         ("threshold", C.c_float), ("topk", C.c_int32), ("ref_mode", C.c_int32),
-        ("score_source", C.c_int32), ("schedule", C.c_int32),
+        ("score_source", C.c_int32), ("schedule", C.c_int32), ("mlp_tokens", C.c_int32),
     ]
 
 
@@ -95,10 +96,11 @@ def set_threads(n: int) -> None:
 
 def make_config(shape, n_streams=1, n_views=1, select_mode=SEL_THRESHOLD, threshold=0.98,
                 topk=0, ref_mode=REF_PREV_FRAME, score_source=SCORE_EMBED,
-                schedule=SCHED_INCREMENTAL) -> OrcConfig:
+                schedule=SCHED_INCREMENTAL, mlp_tokens=MLP_UPDATED) -> OrcConfig:
     return OrcConfig(shape.img_h, shape.img_w, shape.patch, shape.dim, shape.depth,
                      shape.heads, shape.mlp_dim, n_streams, n_views, shape.ln_eps,
-                     shape.gelu, select_mode, threshold, topk, ref_mode, score_source, schedule)
+                     shape.gelu, select_mode, threshold, topk, ref_mode, score_source, schedule,
+                     mlp_tokens)
 
 
 class Oracle:
@@ -106,10 +108,11 @@ class Oracle:
 
     def __init__(self, shape, weights_u16: np.ndarray, n_streams=1, n_views=1,
                  select_mode=SEL_THRESHOLD, threshold=0.98, topk=0,
-                 ref_mode=REF_PREV_FRAME, score_source=SCORE_EMBED, schedule=SCHED_INCREMENTAL):
+                 ref_mode=REF_PREV_FRAME, score_source=SCORE_EMBED, schedule=SCHED_INCREMENTAL,
+                 mlp_tokens=MLP_UPDATED):
         self.shape = shape
         self.cfg = make_config(shape, n_streams, n_views, select_mode, threshold, topk,
-                               ref_mode, score_source, schedule)
+                               ref_mode, score_source, schedule, mlp_tokens)
         self.sv = n_streams * n_views
         self._w = np.ascontiguousarray(weights_u16, dtype=np.uint16)
         self._h = lib().orc_create(C.byref(self.cfg), _p(self._w))
@@ -119,7 +122,8 @@ class Oracle:
     @classmethod
     def for_workload(cls, wl, weights_u16):
         return cls(wl.shape, weights_u16, wl.n_streams, wl.n_views, wl.select_mode,
-                   wl.threshold, wl.topk, wl.ref_mode, wl.score_source, wl.schedule)
+                   wl.threshold, wl.topk, wl.ref_mode, wl.score_source, wl.schedule,
+                   wl.mlp_tokens)
 
     def close(self):
         if self._h:
@@ -160,7 +164,7 @@ class Oracle:
             raise ValueError("bad stream index")
 
     def cache(self, which: str, layer: int = 0) -> np.ndarray:
-        code = {"K": 0, "V": 1, "tokens": 2, "ref": 3}[which]
+        code = {"K": 0, "V": 1, "tokens": 2, "ref": 3, "A": 4}[which]
         out = self._tok()
         if lib().orc_get_cache(self._h, code, int(layer), _p(out)) != 0:
             raise ValueError("bad cache request")

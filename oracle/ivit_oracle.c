@@ -16,9 +16,12 @@
  * Readings where the paper is silent are listed in the repository's design notes:
  * the score compares either the patch embeddings (before the position embedding) or
  * the first layer's keys (Eq. 3 as printed) with their reference; all updated tokens'
- * K/V of a layer are written before that layer's
- * attention; reused tokens' residual streams are never touched; the cached output is
- * the post-final-LN token; a cold view (no reference yet) updates every token.
+ * K/V of a layer are written before that layer's attention; the cached output is the
+ * post-final-LN token; a cold view (no reference yet) updates every token.  Two readings
+ * of what the reused tokens do after attention (mlp_tokens): either their residual
+ * streams are never touched and they keep their cached outputs (0), or they take their
+ * cached attention-block output, and every token goes through the residual addition,
+ * the MLP of every layer and the final LN (1).
  *
  * Precision: fp32 storage, double accumulation of every dot product, LN statistic and
  * softmax sum; the Eq. 3 score in fp32.  OpenMP splits independent output elements
@@ -52,6 +55,7 @@ struct orc_state {
   float* cacheK;  /* [L][SV][N][D] */
   float* cacheV;  /* [L][SV][N][D] */
   float* tok_out; /* [SV][N][D] final tokens (post final LN) */
+  float* cacheA;  /* [L][SV][N][D] attention-block outputs W_o O + b_o (mlp_tokens = 1) */
   uint8_t* cold;  /* [SV] */
 };
 
@@ -296,12 +300,95 @@ static void encode_rows(orc_state* s, int v, const int32_t* U, int m) {
   free(hid);
 }
 
+/* mlp_tokens = 1: runs every block on view v with attention for the updated tokens U
+ * (ascending, m entries) only.  Reused tokens' keys and values come from the cache
+ * (Eq. 5) and so do their attention-block outputs; after the residual addition every
+ * token of the view goes through LN2 and the MLP, and every token's final LN output
+ * is written. */
+static void encode_rows_all(orc_state* s, int v, const int32_t* U, int m) {
+  const int N = s->N, D = s->D, F = s->F, H = s->H, dh = s->dh, SV = s->SV;
+  const float eps = s->cfg.ln_eps;
+  const float* e_t = s->e_t + (size_t)v * N * D;
+  const int mq = m > 0 ? m : 1;
+  float* x = (float*)malloc(sizeof(float) * (size_t)N * D);      /* every token */
+  float* xn = (float*)malloc(sizeof(float) * (size_t)N * D);
+  float* qkv = (float*)malloc(sizeof(float) * (size_t)mq * 3 * D); /* updated tokens */
+  float* att = (float*)malloc(sizeof(float) * (size_t)mq * D);
+  float* a = (float*)malloc(sizeof(float) * (size_t)mq * D);
+  float* hid = (float*)malloc(sizeof(float) * (size_t)N * F);
+
+  /* every token enters the first block: patch embedding + position embedding */
+  for (size_t t = 0; t < (size_t)N * D; ++t) x[t] = e_t[t] + s->pos[t];
+
+  for (int l = 0; l < s->L; ++l) {
+    const orc_layer* w = &s->layer[l];
+    float* Kl = s->cacheK + ((size_t)l * SV + v) * N * D;
+    float* Vl = s->cacheV + ((size_t)l * SV + v) * N * D;
+    float* Al = s->cacheA + ((size_t)l * SV + v) * N * D;
+
+    if (m > 0) {
+      /* Eq. 4 for the updated tokens */
+#pragma omp parallel for schedule(static)
+      for (int r = 0; r < m; ++r)
+        orc_layernorm(x + (size_t)U[r] * D, w->ln1_g, w->ln1_b, D, eps, xn + (size_t)r * D);
+      linear_rows(xn, w->W_qkv, w->b_qkv, m, D, 3 * D, qkv, 0);
+      /* Eq. 5 */
+      for (int r = 0; r < m; ++r) {
+        memcpy(Kl + (size_t)U[r] * D, qkv + (size_t)r * 3 * D + D, sizeof(float) * D);
+        memcpy(Vl + (size_t)U[r] * D, qkv + (size_t)r * 3 * D + 2 * D, sizeof(float) * D);
+      }
+      /* attention for the updated tokens over all N tokens */
+#pragma omp parallel for collapse(2) schedule(static)
+      for (int r = 0; r < m; ++r)
+        for (int h = 0; h < H; ++h) {
+          double* sc = (double*)malloc(sizeof(double) * (size_t)N);
+          attention_row(qkv + (size_t)r * 3 * D + (size_t)h * dh, Kl + (size_t)h * dh,
+                        Vl + (size_t)h * dh, D, N, dh, sc, att + (size_t)r * D + (size_t)h * dh);
+          free(sc);
+        }
+      /* their attention-block outputs replace the cached ones */
+      linear_rows(att, w->W_o, w->b_o, m, D, D, a, 0);
+      for (int r = 0; r < m; ++r) memcpy(Al + (size_t)U[r] * D, a + (size_t)r * D, sizeof(float) * D);
+    }
+
+    /* residual addition for every token (reused tokens: the cached output) */
+    for (size_t t = 0; t < (size_t)N * D; ++t) x[t] += Al[t];
+
+    /* MLP for every token */
+#pragma omp parallel for schedule(static)
+    for (int i = 0; i < N; ++i)
+      orc_layernorm(x + (size_t)i * D, w->ln2_g, w->ln2_b, D, eps, xn + (size_t)i * D);
+    linear_rows(xn, w->W_1, w->b_1, N, D, F, hid, 0);
+#pragma omp parallel for schedule(static)
+    for (size_t t = 0; t < (size_t)N * F; ++t) hid[t] = orc_gelu(hid[t], s->cfg.gelu);
+    linear_rows(hid, w->W_2, w->b_2, N, F, D, x, 1);
+  }
+
+  for (int i = 0; i < N; ++i)
+    orc_layernorm(x + (size_t)i * D, s->lnf_g, s->lnf_b, D, eps, s->tok_out + ((size_t)v * N + i) * D);
+
+  free(x);
+  free(xn);
+  free(qkv);
+  free(att);
+  free(a);
+  free(hid);
+}
+
+static void encode_view(orc_state* s, int v, const int32_t* U, int m) {
+  if (s->cfg.mlp_tokens == 1)
+    encode_rows_all(s, v, U, m);
+  else
+    encode_rows(s, v, U, m);
+}
+
 orc_state* orc_create(const orc_config* cfg, const uint16_t* wb) {
   if (!cfg || !wb) return NULL;
   if (cfg->patch <= 0 || cfg->img_h % cfg->patch || cfg->img_w % cfg->patch) return NULL;
   if (cfg->dim <= 0 || cfg->heads <= 0 || cfg->dim % cfg->heads || cfg->depth <= 0 ||
       cfg->mlp_dim <= 0 || cfg->n_streams <= 0 || cfg->n_views <= 0)
     return NULL;
+  if (cfg->mlp_tokens != 0 && cfg->mlp_tokens != 1) return NULL;
   orc_state* s = (orc_state*)calloc(1, sizeof(orc_state));
   s->cfg = *cfg;
   s->N = (cfg->img_h / cfg->patch) * (cfg->img_w / cfg->patch);
@@ -346,8 +433,10 @@ orc_state* orc_create(const orc_config* cfg, const uint16_t* wb) {
   s->tok_out = (float*)calloc(view, sizeof(float));
   s->cacheK = (float*)calloc(view * s->L, sizeof(float));
   s->cacheV = (float*)calloc(view * s->L, sizeof(float));
+  s->cacheA = cfg->mlp_tokens == 1 ? (float*)calloc(view * s->L, sizeof(float)) : NULL;
   s->cold = (uint8_t*)malloc((size_t)s->SV);
-  if (!s->e_ref || !s->e_t || !s->s_t || !s->tok_out || !s->cacheK || !s->cacheV || !s->cold) {
+  if (!s->e_ref || !s->e_t || !s->s_t || !s->tok_out || !s->cacheK || !s->cacheV || !s->cold ||
+      (cfg->mlp_tokens == 1 && !s->cacheA)) {
     orc_destroy(s);
     return NULL;
   }
@@ -365,6 +454,7 @@ void orc_destroy(orc_state* s) {
   free(s->tok_out);
   free(s->cacheK);
   free(s->cacheV);
+  free(s->cacheA);
   free(s->cold);
   free(s);
 }
@@ -401,7 +491,7 @@ int orc_encode_full(orc_state* s, const uint8_t* frames, float* tokens_out) {
   for (int v = 0; v < s->SV; ++v) {
     memcpy(s->e_ref + (size_t)v * N * D, score_vectors(s) + (size_t)v * N * D,
            sizeof(float) * (size_t)N * D);
-    encode_rows(s, v, U, N);
+    encode_view(s, v, U, N);
     s->cold[v] = 0;
   }
   free(U);
@@ -451,7 +541,7 @@ int orc_encode_incremental(orc_state* s, const uint8_t* frames, float* tokens_ou
       for (int r = 0; r < m; ++r)
         memcpy(er + (size_t)U[r] * D, et + (size_t)U[r] * D, sizeof(float) * D);
     }
-    encode_rows(s, v, U, m);
+    encode_view(s, v, U, m);
     s->cold[v] = 0;
     if (counts_out) counts_out[v] = m;
     if (idx_out)
@@ -483,6 +573,9 @@ int orc_get_cache(const orc_state* s, int which, int layer, float* out) {
     src = s->tok_out;
   } else if (which == 3) {
     src = s->e_ref;
+  } else if (which == 4 && s->cacheA) {
+    if (layer < 0 || layer >= s->L) return -1;
+    src = s->cacheA + (size_t)layer * view;
   } else {
     return -1;
   }

@@ -39,6 +39,11 @@ typedef struct orc_config {
                            1: first-layer keys (Eq. 3) */
   int32_t schedule;     /* 0: every incremental call is incremental,
                            1: odd/even chunks (odd calls encode in full, Sec. III-B) */
+  int32_t mlp_tokens;   /* 0: the blocks run on the updated tokens only (reused tokens keep
+                           their cached outputs); 1: attention runs on the updated tokens,
+                           reused tokens take their cached attention outputs, and every
+                           token goes through the residual addition and the MLP of every
+                           layer (Sec. III-B, the passage after Eq. 5) */
 } orc_config;
 
 typedef struct orc_state orc_state;
@@ -64,7 +69,8 @@ int orc_reset(orc_state* s, int stream);
 
 /* Cache read-out for tests.  which: 0 = K, 1 = V (layer `layer`), 2 = final tokens,
  * 3 = reference score vectors (patch embeddings or first-layer keys, per
- * score_source).  out: float [S*V][N][D]. */
+ * score_source), 4 = attention-block outputs W_o O + b_o of layer `layer` (mlp_tokens
+ * = 1 only).  out: float [S*V][N][D]. */
 int orc_get_cache(const orc_state* s, int which, int layer, float* out);
 
 /* ---- building blocks (each a step of the method, exported for pinning) ---- */

@@ -379,6 +379,7 @@ class Workload:
     ref_mode: int = REF_PREV_FRAME
     score_source: int = SCORE_EMBED
     schedule: int = SCHED_INCREMENTAL
+    mlp_tokens: int = 0  # 0: blocks on the updated tokens only; 1: MLP on every token
     scene: str = "rects"
     views: Tuple[ViewScene, ...] = field(default_factory=tuple)
     repaint_k: int = 0

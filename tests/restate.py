@@ -83,3 +83,35 @@ def layer0_keys(shape, W, e):
     xn = F.layer_norm(e + W["pos"], (D,), W["l0.ln1_g"], W["l0.ln1_b"], shape.ln_eps)
     xn = xn.float().bfloat16().double()
     return F.linear(xn, W["l0.W_qkv"][D:2 * D], W["l0.b_qkv"][D:2 * D])
+
+
+def run_rows_mlp_all(shape, W, e, mask, K, V, A):
+    """The MLP-on-all-tokens reading (Sec. III-B, after Eq. 5): attention for the tokens
+    where ``mask`` is true only (their K/V and attention-block outputs replace the cached
+    ones in K, V, A [L, N, D]); every token then takes the residual addition with its
+    attention-block output (cached for reused tokens), LN2 + MLP, and the final LN.
+    Returns (K, V, A, tokens [N, D]) as new tensors."""
+    D, H, eps = shape.dim, shape.heads, shape.ln_eps
+    K, V, A = K.clone(), V.clone(), A.clone()
+    sel = torch.nonzero(torch.as_tensor(mask)).flatten()
+    x = e + W["pos"]
+    for l in range(shape.depth):
+        p = lambda n: W[f"l{l}.{n}"]
+        xn = F.layer_norm(x[sel], (D,), p("ln1_g"), p("ln1_b"), eps)
+        q, k, v = F.linear(xn, p("W_qkv"), p("b_qkv")).split(D, dim=1)
+        K[l] = K[l].index_put((sel,), k)
+        V[l] = V[l].index_put((sel,), v)
+        A[l] = A[l].index_put((sel,), F.linear(_attend(q, K[l], V[l], H), p("W_o"), p("b_o")))
+        x = x + A[l]
+        x = x + F.linear(_gelu(F.linear(F.layer_norm(x, (D,), p("ln2_g"), p("ln2_b"), eps),
+                                        p("W_1"), p("b_1")), shape), p("W_2"), p("b_2"))
+    return K, V, A, F.layer_norm(x, (D,), W["lnf_g"], W["lnf_b"], eps)
+
+
+def full_mlp_all(shape, W, frame):
+    """Full encode under the MLP-on-all-tokens reading: (tokens, K, V, A, e)."""
+    N, D, L = shape.n_tokens, shape.dim, shape.depth
+    e = embed(shape, W, frame)
+    Z = torch.zeros(L, N, D, dtype=torch.float64)
+    K, V, A, tok = run_rows_mlp_all(shape, W, e, torch.ones(N, dtype=torch.bool), Z, Z, Z)
+    return tok, K, V, A, e
