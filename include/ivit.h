@@ -50,6 +50,8 @@ extern "C" {
 #define IVIT_SCORE_KEY0 1      /* Eq. 3 as printed: first-layer keys W_K LN1(e+pos) + b_K */
 #define IVIT_SCHED_INCREMENTAL 0 /* every ivit_encode_incremental call is incremental */
 #define IVIT_SCHED_ODD_EVEN 1  /* odd calls encode in full, even calls incrementally */
+#define IVIT_MLP_UPDATED 0     /* every block runs on the updated tokens only */
+#define IVIT_MLP_ALL 1         /* attention on the updated tokens, residual + MLP on all */
 
 /* Encoder + selection configuration.
  * Supported by the kernels: patch >= 1 dividing img_h and img_w; N <= 1024;
@@ -72,6 +74,12 @@ typedef struct ivit_config {
   int32_t ref_mode;      /* IVIT_REF_* */
   int32_t score_source;  /* IVIT_SCORE_*: what Eq. 3's cosine compares (Sec. III-B) */
   int32_t schedule;      /* IVIT_SCHED_*: odd/even chunking of Sec. III-B, or none */
+  int32_t mlp_tokens;    /* IVIT_MLP_*: which tokens go through the residual addition and
+                            the MLP after attention (Sec. III-B, the passage after Eq. 5).
+                            IVIT_MLP_ALL keeps every token's attention-block output
+                            W_o O + b_o per layer (fp32 [L][SV][N][D]); reused tokens take
+                            theirs from that cache, every token runs LN2 + MLP and the
+                            final LN, and every output token is recomputed. */
 } ivit_config;
 
 typedef struct ivit_handle ivit_handle;
@@ -108,7 +116,9 @@ int ivit_encode_full(ivit_handle* h, const uint8_t* frames_dev, uint16_t* tokens
  * recomputed, the rest from the final-token cache.  A cold view updates every token.
  * tokens_out_dev: bf16 [SV][N][D] or NULL.  changed_count_dev: int32 [SV] number of
  * updated tokens per view, or NULL.  No host synchronisation happens inside.  With
- * schedule = IVIT_SCHED_ODD_EVEN the 1st, 3rd, ... call encodes in full (count N). */
+ * schedule = IVIT_SCHED_ODD_EVEN the 1st, 3rd, ... call encodes in full (count N).
+ * With mlp_tokens = IVIT_MLP_ALL the blocks after attention run on every token (see
+ * ivit_config). */
 int ivit_encode_incremental(ivit_handle* h, const uint8_t* frames_dev,
                             uint16_t* tokens_out_dev, int32_t* changed_count_dev,
                             void* stream);
@@ -121,8 +131,9 @@ int ivit_get_changed(ivit_handle* h, int sv, int32_t* idx_dev, int32_t* count_de
 
 /* Copies per-view state for inspection: which = 0 key cache of `layer`, 1 value cache
  * of `layer`, 2 final-token cache (all bf16 [SV][N][D]), 3 reference score vectors
- * (patch embeddings or first-layer keys, fp32 [SV][N][D]).  dst_dev must hold that many
- * bytes. */
+ * (patch embeddings or first-layer keys, fp32 [SV][N][D]), 4 attention-block outputs of
+ * `layer` (fp32 [SV][N][D], mlp_tokens = IVIT_MLP_ALL only).  dst_dev must hold that
+ * many bytes. */
 int ivit_get_cache(ivit_handle* h, int which, int layer, void* dst_dev, void* stream);
 
 /* Marks the views of camera stream `stream_index` (all streams if -1) cold: the next

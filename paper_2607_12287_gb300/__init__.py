@@ -41,7 +41,7 @@ class IvitConfig(C.Structure):
         ("mlp_dim", C.c_int32), ("n_streams", C.c_int32), ("n_views", C.c_int32),
         ("ln_eps", C.c_float), ("gelu", C.c_int32), ("select_mode", C.c_int32),
         ("threshold", C.c_float), ("topk", C.c_int32), ("ref_mode", C.c_int32),
-        ("score_source", C.c_int32), ("schedule", C.c_int32),
+        ("score_source", C.c_int32), ("schedule", C.c_int32), ("mlp_tokens", C.c_int32),
     ]
 
 
@@ -109,10 +109,10 @@ def _stream(stream) -> Optional[int]:
 def make_config(shape: "synth.EncoderShape", n_streams: int = 1, n_views: int = 1,
                 select_mode: int = synth.SEL_THRESHOLD, threshold: float = 0.98, topk: int = 0,
                 ref_mode: int = synth.REF_PREV_FRAME, score_source: int = synth.SCORE_EMBED,
-                schedule: int = synth.SCHED_INCREMENTAL) -> IvitConfig:
+                schedule: int = synth.SCHED_INCREMENTAL, mlp_tokens: int = 0) -> IvitConfig:
     return IvitConfig(shape.img_h, shape.img_w, shape.patch, shape.dim, shape.depth, shape.heads,
                       shape.mlp_dim, n_streams, n_views, shape.ln_eps, shape.gelu, select_mode,
-                      threshold, topk, ref_mode, score_source, schedule)
+                      threshold, topk, ref_mode, score_source, schedule, mlp_tokens)
 
 
 # ------------------------------------------------------------- C entry points
@@ -199,20 +199,21 @@ class IncrementalViT:
     def __init__(self, shape: "synth.EncoderShape", weights_u16: np.ndarray, n_streams: int = 1,
                  n_views: int = 1, select_mode: int = synth.SEL_THRESHOLD,
                  threshold: float = 0.98, topk: int = 0, ref_mode: int = synth.REF_PREV_FRAME,
-                 score_source: int = synth.SCORE_EMBED, schedule: int = synth.SCHED_INCREMENTAL):
+                 score_source: int = synth.SCORE_EMBED, schedule: int = synth.SCHED_INCREMENTAL,
+                 mlp_tokens: int = 0):
         import torch
         self.torch = torch
         self.shape = shape
         self.sv = n_streams * n_views
         self.cfg = make_config(shape, n_streams, n_views, select_mode, threshold, topk, ref_mode,
-                               score_source, schedule)
+                               score_source, schedule, mlp_tokens)
         self.h = ivit_create(self.cfg, weights_u16)
         self.device = torch.device("cuda", torch.cuda.current_device())
 
     @classmethod
     def for_workload(cls, wl, weights_u16):
         return cls(wl.shape, weights_u16, wl.n_streams, wl.n_views, wl.select_mode, wl.threshold,
-                   wl.topk, wl.ref_mode, wl.score_source, wl.schedule)
+                   wl.topk, wl.ref_mode, wl.score_source, wl.schedule, wl.mlp_tokens)
 
     def close(self):
         if getattr(self, "h", None):
@@ -248,8 +249,8 @@ class IncrementalViT:
         return idx[: int(cnt.item())]
 
     def cache(self, which: str, layer: int = 0, stream=None):
-        code = {"K": 0, "V": 1, "tokens": 2, "ref": 3}[which]
-        dt = self.torch.float32 if code == 3 else self.torch.bfloat16
+        code = {"K": 0, "V": 1, "tokens": 2, "ref": 3, "A": 4}[which]
+        dt = self.torch.float32 if code in (3, 4) else self.torch.bfloat16
         dst = self.torch.empty((self.sv, self.shape.n_tokens, self.shape.dim), dtype=dt,
                                device=self.device)
         ivit_get_cache(self.h, code, layer, dst, stream)

@@ -119,6 +119,7 @@ struct ivit_handle {
   bf16* patches = nullptr;
   float *e_t = nullptr, *e_ref = nullptr, *sims = nullptr, *x = nullptr;
   float* key_t = nullptr;          // first-layer keys of every token (score_source KEY0)
+  float* acache = nullptr;         // [L][M_max][D] attention-block outputs (mlp_tokens ALL)
   int* rowtok_all = nullptr;       // identity row -> token map, all SV*N rows
   int* m_all = nullptr;            // device copy of SV*N
   CUtensorMap tm_wk0;              // layer 0's key projection (rows D..2D-1 of W_qkv)
@@ -196,6 +197,7 @@ const char* validate(const ivit_config* c) {
   if (!std::isfinite(c->threshold)) return "threshold must be finite";
   if (c->score_source != IVIT_SCORE_EMBED && c->score_source != IVIT_SCORE_KEY0) return "bad score_source";
   if (c->schedule != IVIT_SCHED_INCREMENTAL && c->schedule != IVIT_SCHED_ODD_EVEN) return "bad schedule";
+  if (c->mlp_tokens != IVIT_MLP_UPDATED && c->mlp_tokens != IVIT_MLP_ALL) return "bad mlp_tokens";
   return nullptr;
 }
 
@@ -238,6 +240,7 @@ int setup_persistent(ivit_handle* h) {
   // Default: small encoders (dim <= 384), whose per-layer kernels are launch-bound.
   const char* path = std::getenv("IVIT_PATH");
   if (path && std::strcmp(path, "kernels") == 0) return IVIT_OK;
+  if (h->cfg.mlp_tokens == IVIT_MLP_ALL) return IVIT_OK;  // the kernel chain runs that reading
   if (!(path && std::strcmp(path, "persistent") == 0) && h->D > 384) return IVIT_OK;
   const int dh = h->D / h->H;
   const size_t smem = ivit::persistent_smem_bytes(h->N, dh);
@@ -483,6 +486,7 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   const size_t o_ck = sa.take(L * M * D * 2), o_cv = sa.take(L * M * D * 2), o_tok = sa.take(M * D * 2);
   const size_t o_err = sa.take(4);
   const size_t o_key = c.score_source == IVIT_SCORE_KEY0 ? sa.take(M * D * 4) : 0;
+  const size_t o_acache = c.mlp_tokens == IVIT_MLP_ALL ? sa.take(L * M * D * 4) : 0;
   const size_t o_rta = sa.take(M * 4), o_mall = sa.take(4);
   const size_t o_fb = sa.take(static_cast<size_t>(h->SV) * c.img_h * c.img_w * 3);
   const size_t o_cb = sa.take(h->SV * 4);
@@ -508,6 +512,7 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   h->tok_out = sa.at<bf16>(o_tok);
   h->err = sa.at<int>(o_err);
   if (c.score_source == IVIT_SCORE_KEY0) h->key_t = sa.at<float>(o_key);
+  if (c.mlp_tokens == IVIT_MLP_ALL) h->acache = sa.at<float>(o_acache);
   h->rowtok_all = sa.at<int>(o_rta);
   h->m_all = sa.at<int>(o_mall);
   {
@@ -614,6 +619,114 @@ void print_trace(ivit_handle* h, cudaStream_t s) {
     if (cnt[k]) std::fprintf(stderr, "  %-12s %6.2f us x %d\n", names[k], acc[k] / cnt[k], cnt[k]);
 }
 
+// Attention of the updated queries over all tokens of their view for one layer.
+int attention(ivit_handle* h, const LayerW& w, const bf16* ck, const bf16* cv, bool full, cudaStream_t s) {
+  const int N = h->N, D = h->D, SV = h->SV;
+  if (h->attn_tc) {
+    ivit::AttnTcArgs at;
+    at.cache_k = ck;
+    at.cache_v = cv;
+    at.cu_rows = h->cu_rows;
+    at.rowtok = h->rowtok;
+    at.o = h->o;
+    at.err = h->err;
+    at.n_tok = N;
+    at.dim = D;
+    at.dh = D / h->H;
+    at.heads = h->H;
+    at.sv = SV;
+    at.qtiles = (N + 127) / 128;
+    at.prefetch = full ? 0 : 1;
+    at.key_splits = full ? h->attn_splits_full : h->attn_splits_inc;
+    IVIT_CK(h, ivit::launch_attention_tc(h->tm_qa, w.tm_ak, w.tm_av, at, h->num_sms, s));
+  } else {
+    IVIT_CK(h, ivit::launch_attention(w.tm_ck, w.tm_cv, h->q, ck, cv, h->cu_rows, h->rowtok, h->o, SV, N, D, h->H,
+                                      full ? (N + 31) / 32 : std::max(1, (N / 10 + 31) / 32), s));
+  }
+  ++h->launches;
+  return IVIT_OK;
+}
+
+// The blocks under the MLP-on-all-tokens reading (Sec. III-B, after Eq. 5): x holds
+// every token's residual stream (row = token v*N + i).  Per layer, the updated tokens
+// (packed rows, rowtok) run LN1, QKV with the K/V scatter (Eq. 5), attention over all
+// tokens and the output projection, whose result replaces their rows of the layer's
+// attention-output cache; then every token adds its cached attention output to its
+// stream (fused into LN2) and runs the MLP; the final LN writes every output token.
+int run_layers_mlp_all(ivit_handle* h, const GemmPlan* plan, bool full, cudaStream_t s) {
+  const ivit_config& c = h->cfg;
+  const int N = h->N, D = h->D, F = h->F, SV = h->SV, M = h->M_max;
+  const int* total = h->cu_rows + SV;
+  for (int l = 0; l < h->L; ++l) {
+    const LayerW& w = h->layers[l];
+    bf16* ck = h->cacheK + static_cast<size_t>(l) * M * D;
+    bf16* cv = h->cacheV + static_cast<size_t>(l) * M * D;
+    float* al = h->acache + static_cast<size_t>(l) * M * D;
+    IVIT_CK(h, ivit::launch_layernorm_ex(total, h->x, nullptr, h->rowtok, w.ln1g, w.ln1b, h->xn, nullptr, D,
+                                         c.ln_eps, M, h->row_grid, s));
+    ++h->launches;
+    {
+      ivit::GemmArgs a;
+      a.n_out = 3 * D;
+      a.k = D;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiQKV;
+      a.epi.bias = w.bqkv;
+      a.epi.out_bf16 = h->q;
+      a.epi.ld_out = D;
+      a.epi.cache_k = ck;
+      a.epi.cache_v = cv;
+      a.epi.rowtok = h->rowtok;
+      a.epi.dim = D;
+      if (int r = gemm(h, plan[kGemmQKV], w.tm_qkv, h->tm_xn, a, s)) return r;
+    }
+    if (int r = attention(h, w, ck, cv, full, s)) return r;
+    {
+      ivit::GemmArgs a;
+      a.n_out = D;
+      a.k = D;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiScatterF32;
+      a.epi.bias = w.bo;
+      a.epi.out_f32 = al;
+      a.epi.ld_out = D;
+      a.epi.rowtok = h->rowtok;
+      if (int r = gemm(h, plan[kGemmO], w.tm_o, h->tm_o, a, s)) return r;
+    }
+    IVIT_CK(h, ivit::launch_layernorm_ex(h->m_all, h->x, al, nullptr, w.ln2g, w.ln2b, h->xn, nullptr, D, c.ln_eps,
+                                         M, h->row_grid, s));
+    ++h->launches;
+    {
+      ivit::GemmArgs a;
+      a.n_out = F;
+      a.k = D;
+      a.m_static = M;
+      a.epi.kind = ivit::kEpiGelu;
+      a.epi.bias = w.b1;
+      a.epi.out_bf16 = h->hbuf;
+      a.epi.ld_out = F;
+      a.epi.gelu_mode = c.gelu;
+      if (int r = gemm(h, h->plan_full[kGemmUp], w.tm_1, h->tm_xn, a, s)) return r;
+    }
+    {
+      ivit::GemmArgs a;
+      a.n_out = D;
+      a.k = F;
+      a.m_static = M;
+      a.epi.kind = ivit::kEpiResid;
+      a.epi.bias = w.b2;
+      a.epi.out_f32 = h->x;
+      a.epi.ld_out = D;
+      if (int r = gemm(h, h->plan_full[kGemmDown], w.tm_2, h->tm_h, a, s)) return r;
+    }
+  }
+  IVIT_CK(h, ivit::launch_layernorm(h->m_all, h->x, h->lnfg, h->lnfb, h->tok_out, nullptr, D, c.ln_eps, M,
+                                    h->row_grid, s));
+  ++h->launches;
+  (void)N;
+  return IVIT_OK;
+}
+
 // Enqueues the whole chain for one frame per view on `s` (eagerly or under capture).
 int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool full, cudaStream_t s) {
   const ivit_config& c = h->cfg;
@@ -669,6 +782,16 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
                                  c.topk, cm, h->idx, h->counts, h->cu_rows, h->rowtok, h->done_ctr,
                                  user_counts, s));
   ++h->launches;
+  if (c.mlp_tokens == IVIT_MLP_ALL) {
+    // every token's residual stream (token-indexed), then the references of the updated
+    // tokens (last-refresh mode, cold views) without touching x
+    IVIT_CK(h, ivit::launch_gather(h->m_all, h->rowtok_all, h->e_t, h->pos, h->x, nullptr, h->e_ref, N, D, 0,
+                                   cm, M, h->row_grid, s));
+    IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, nullptr, score_vec, h->e_ref, N, D,
+                                   c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
+    h->launches += 2;
+    return run_layers_mlp_all(h, plan, full, s);
+  }
   IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, h->x, score_vec, h->e_ref, N, D,
                                  c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
   ++h->launches;
@@ -706,28 +829,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
       a.epi.dim = D;
       if (int r = gemm(h, plan[kGemmQKV], w.tm_qkv, h->tm_xn, a, s)) return r;
     }
-    if (h->attn_tc) {
-      ivit::AttnTcArgs at;
-      at.cache_k = ck;
-      at.cache_v = cv;
-      at.cu_rows = h->cu_rows;
-      at.rowtok = h->rowtok;
-      at.o = h->o;
-      at.err = h->err;
-      at.n_tok = N;
-      at.dim = D;
-      at.dh = D / h->H;
-      at.heads = h->H;
-      at.sv = SV;
-      at.qtiles = (N + 127) / 128;
-      at.prefetch = full ? 0 : 1;
-      at.key_splits = full ? h->attn_splits_full : h->attn_splits_inc;
-      IVIT_CK(h, ivit::launch_attention_tc(h->tm_qa, w.tm_ak, w.tm_av, at, h->num_sms, s));
-    } else {
-      IVIT_CK(h, ivit::launch_attention(w.tm_ck, w.tm_cv, h->q, ck, cv, h->cu_rows, h->rowtok, h->o, SV, N, D,
-                                        h->H, full ? (N + 31) / 32 : std::max(1, (N / 10 + 31) / 32), s));
-    }
-    ++h->launches;
+    if (int r = attention(h, w, ck, cv, full, s)) return r;
     {
       ivit::GemmArgs a;
       a.n_out = D;
@@ -907,6 +1009,10 @@ int ivit_get_cache(ivit_handle* h, int which, int layer, void* dst_dev, void* st
     src = h->tok_out;
   } else if (which == 3) {
     src = h->e_ref;
+    bytes = elems * 4;
+  } else if (which == 4 && h->acache) {
+    if (layer < 0 || layer >= h->L) return h->fail(IVIT_ERR_ARG, "layer out of range");
+    src = h->acache + static_cast<size_t>(layer) * elems;
     bytes = elems * 4;
   } else {
     return h->fail(IVIT_ERR_ARG, "bad cache selector");

@@ -58,6 +58,9 @@ __device__ __forceinline__ void epilogue_store(const GemmEpilogue& e, int r, int
     case kEpiGelu:
       e.out_bf16[static_cast<size_t>(r) * e.ld_out + f] = __float2bfloat16_rn(gelu_f(val, e.gelu_mode));
       break;
+    case kEpiScatterF32:
+      e.out_f32[static_cast<size_t>(e.rowtok[r]) * e.ld_out + f] = val;
+      break;
     default: {  // kEpiQKV
       const int D = e.dim;
       if (f < D) {

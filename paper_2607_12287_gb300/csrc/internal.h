@@ -52,6 +52,7 @@ enum EpiKind : int {
                     // f < 2D: cache_k[rowtok[r]][f-D], else cache_v[rowtok[r]][f-2D]  (Eq. 5)
   kEpiResid = 2,    // out_f32[r][f] += y + bias[f]  (residual stream, fp32)
   kEpiGelu = 3,     // out_bf16[r][f] = gelu(y + bias[f])
+  kEpiScatterF32 = 4,  // out_f32[rowtok[r]][f] = y + bias[f]  (per-token output cache)
 };
 
 struct GemmEpilogue {
@@ -145,6 +146,11 @@ cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const flo
 cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma, const float* beta,
                              bf16* y, const int* dst_rowtok, int dim, float eps, int max_rows,
                              int grid, cudaStream_t s);
+// The same, reading row src_rowtok[r] of x when src_rowtok is set, and when `add` is set
+// first adding row src_rowtok[r] (or r) of `add` to x in place: x += add; y = LN(x).
+cudaError_t launch_layernorm_ex(const int* rows, float* x, const float* add, const int* src_rowtok,
+                                const float* gamma, const float* beta, bf16* y, const int* dst_rowtok, int dim,
+                                float eps, int max_rows, int grid, cudaStream_t s);
 
 // One-time function attributes of the attention kernel (dynamic shared memory opt-in).
 cudaError_t attention_setup();

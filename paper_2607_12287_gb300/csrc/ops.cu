@@ -185,10 +185,12 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
     const bool refresh = ref_src && (ref_last_refresh || is_cold(cold, tok / N));
     const float4* a = reinterpret_cast<const float4*>(e_t + static_cast<size_t>(tok) * dim);
     const float4* p = reinterpret_cast<const float4*>(pos + static_cast<size_t>(ti) * dim);
-    float4* y = reinterpret_cast<float4*>(x + static_cast<size_t>(r) * dim);
-    for (int c = lane; c < dim / 4; c += 32) {
-      const float4 u = a[c], w = p[c];
-      y[c] = make_float4(u.x + w.x, u.y + w.y, u.z + w.z, u.w + w.w);
+    if (x) {  // (a call that only refreshes references passes no x)
+      float4* y = reinterpret_cast<float4*>(x + static_cast<size_t>(r) * dim);
+      for (int c = lane; c < dim / 4; c += 32) {
+        const float4 u = a[c], w = p[c];
+        y[c] = make_float4(u.x + w.x, u.y + w.y, u.z + w.z, u.w + w.w);
+      }
     }
     if (refresh) {
       const float4* src = reinterpret_cast<const float4*>(ref_src + static_cast<size_t>(tok) * dim);
@@ -204,7 +206,12 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
 // from registers in fp32.
 constexpr int LN_MAX_F4_PER_LANE = 16;
 
-__global__ void layernorm_kernel(const int* __restrict__ nrows, const float* __restrict__ x,
+// Optionally the input row is gathered (row src_rowtok[r] of x) and, with kAdd, a
+// second fp32 array is added to it first and the sum written back to x (the residual
+// addition fused into the LN).
+template <bool kAdd, bool kGather>
+__global__ void layernorm_kernel(const int* __restrict__ nrows, float* __restrict__ x,
+                                 const float* __restrict__ add, const int* __restrict__ src_rowtok,
                                  const float* __restrict__ gamma, const float* __restrict__ beta,
                                  bf16* __restrict__ y, const int* __restrict__ dst_rowtok, int dim,
                                  float eps) {
@@ -226,13 +233,19 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, const float* __r
   pdl_wait();
   pdl_launch_dependents();
   for (int r = blockIdx.x * warps + (threadIdx.x >> 5); r < rows; r += gridDim.x * warps) {
-    const float4* xr = reinterpret_cast<const float4*>(x + static_cast<size_t>(r) * dim);
+    const size_t irow = kGather ? static_cast<size_t>(src_rowtok[r]) : static_cast<size_t>(r);
+    const float4* xr = reinterpret_cast<const float4*>(static_cast<const float*>(x) + irow * dim);
     float4 v[LN_MAX_F4_PER_LANE];
     float sum = 0.f;
 #pragma unroll
     for (int i = 0; i < LN_MAX_F4_PER_LANE; ++i) {
       const int c = lane + 32 * i;
       v[i] = c < n4 ? xr[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+      if (kAdd && c < n4) {
+        const float4 w = reinterpret_cast<const float4*>(add + irow * dim)[c];
+        v[i] = make_float4(v[i].x + w.x, v[i].y + w.y, v[i].z + w.z, v[i].w + w.w);
+        reinterpret_cast<float4*>(x + irow * dim)[c] = v[i];
+      }
       sum += (v[i].x + v[i].y) + (v[i].z + v[i].w);
     }
     const float mean = warp_sum(sum) / dim;
@@ -515,9 +528,18 @@ cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const flo
 cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma, const float* beta,
                              bf16* y, const int* dst_rowtok, int dim, float eps, int max_rows,
                              int grid, cudaStream_t s) {
+  return launch_layernorm_ex(rows, const_cast<float*>(x), nullptr, nullptr, gamma, beta, y, dst_rowtok, dim, eps,
+                             max_rows, grid, s);
+}
+
+cudaError_t launch_layernorm_ex(const int* rows, float* x, const float* add, const int* src_rowtok,
+                                const float* gamma, const float* beta, bf16* y, const int* dst_rowtok, int dim,
+                                float eps, int max_rows, int grid, cudaStream_t s) {
   grid = max(1, min(grid, (max_rows + 7) / 8));
-  return launch_ex(layernorm_kernel, dim3(grid), dim3(256), 0, s, 1, rows, x, gamma, beta, y, dst_rowtok,
-                   dim, eps);
+  auto kern = add ? (src_rowtok ? layernorm_kernel<true, true> : layernorm_kernel<true, false>)
+                  : (src_rowtok ? layernorm_kernel<false, true> : layernorm_kernel<false, false>);
+  return launch_ex(kern, dim3(grid), dim3(256), 0, s, 1, rows, x, add, src_rowtok, gamma, beta, y, dst_rowtok, dim,
+                   eps);
 }
 
 size_t attention_smem(int dh) {

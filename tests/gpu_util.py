@@ -31,15 +31,15 @@ def assert_tokens_close(gpu: np.ndarray, ref: np.ndarray, what: str = ""):
 
 def run_side_by_side(pkg, oracle_mod, shape, weights, frames, n_streams=1, n_views=1,
                      select_mode=0, threshold=0.98, topk=0, ref_mode=0, margin=2e-3,
-                     check_caches=False, first_full=True, score_source=0, schedule=0):
+                     check_caches=False, first_full=True, score_source=0, schedule=0, mlp_tokens=0):
     """Feeds ``frames`` (list of uint8 [SV,H,W,3]) to both sides; frame 0 is a full
     encode when ``first_full``.  Returns per-frame (rel, cos, counts)."""
     import torch
 
     enc = pkg.IncrementalViT(shape, weights, n_streams, n_views, select_mode, threshold, topk,
-                             ref_mode, score_source, schedule)
+                             ref_mode, score_source, schedule, mlp_tokens)
     orc = oracle_mod.Oracle(shape, weights, n_streams, n_views, select_mode, threshold, topk,
-                            ref_mode, score_source, schedule)
+                            ref_mode, score_source, schedule, mlp_tokens)
     sv = n_streams * n_views
     stats = []
     try:
@@ -71,7 +71,7 @@ def run_side_by_side(pkg, oracle_mod, shape, weights, frames, n_streams=1, n_vie
             stats.append((rel, cos, counts))
         if check_caches:
             for l in (0, shape.depth - 1):
-                for which in ("K", "V"):
+                for which in ("K", "V", "A") if mlp_tokens else ("K", "V"):
                     g = enc.cache(which, l).float().cpu().numpy()
                     r = orc.cache(which, l)
                     assert_tokens_close(g, r, f"cache {which} layer {l}")

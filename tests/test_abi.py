@@ -47,6 +47,7 @@ def test_weights_size_matches_generator_layout(pkg):
 @pytest.mark.parametrize("field,value", [
     ("dim", 100), ("heads", 7), ("patch", 15), ("mlp_dim", 1001), ("depth", 0),
     ("n_views", 0), ("gelu", 5), ("select_mode", 9), ("ref_mode", 3), ("ln_eps", 0.0),
+    ("score_source", 2), ("schedule", 4), ("mlp_tokens", 2),
 ])
 def test_bad_config_rejected_before_device_work(pkg, field, value):
     cfg = pkg.make_config(synth.SO400M_224)

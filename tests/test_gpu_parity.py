@@ -179,3 +179,48 @@ def test_odd_even_schedule(pkg, oracle_mod):
     N = shape.n_tokens
     assert [s[2].tolist() for s in stats[0::2]] == [[N, N]] * 3
     assert all(s[2].max() < N for s in stats[1::2])
+
+
+# ---- the MLP-on-all-tokens reading (attention for updated tokens, MLP for every token)
+
+@pytest.mark.parametrize("shape,S,V", [(SHAPE_A, 1, 3), (SHAPE_B, 2, 1), (SHAPE_C, 1, 2)],
+                         ids=["A_d320_3view", "B_n196_2stream", "C_dh72"])
+def test_mlp_all_tokens(pkg, oracle_mod, shape, S, V):
+    w = synth.make_weights(shape, 105)
+    frames = list(synth.stream_random(shape, S * V, 4, 106, change_p=0.2))
+    # +-1 noise on every pixel of the later frames: reused tokens' streams move too
+    rng = np.random.Generator(np.random.PCG64(107))
+    for t in range(1, len(frames)):
+        noise = rng.integers(-1, 2, size=frames[t].shape)
+        frames[t] = np.clip(frames[t].astype(np.int16) + noise, 0, 255).astype(np.uint8)
+    run_side_by_side(pkg, oracle_mod, shape, w, frames, S, V, check_caches=True, mlp_tokens=1)
+
+
+@pytest.mark.parametrize("mode,k", [(synth.SEL_TOPK, 7), (synth.SEL_THRESHOLD, 0)])
+def test_mlp_all_tokens_topk_last_refresh_cold(pkg, oracle_mod, mode, k):
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 111)
+    frames = list(synth.stream_repaint(shape, 2, 4, k or 5, 112))
+    run_side_by_side(pkg, oracle_mod, shape, w, frames, 1, 2, select_mode=mode, topk=k,
+                     ref_mode=synth.REF_LAST_REFRESH, first_full=False, mlp_tokens=1)
+
+
+def test_mlp_all_tokens_identical_frames(pkg, oracle_mod):
+    import torch
+    shape = SHAPE_C
+    w = synth.make_weights(shape, 121)
+    f0 = next(synth.stream_random(shape, 2, 1, 122))
+    enc = pkg.IncrementalViT(shape, w, 1, 2, mlp_tokens=1)
+    try:
+        fd = torch.from_numpy(f0).cuda()
+        t0 = enc.encode_full(fd).clone()
+        t1, cnt = enc.encode_incremental(fd)
+        assert cnt.cpu().numpy().tolist() == [0, 0]
+        # every token is recomputed from the same stream and cached attention outputs,
+        # with the full encode's MLP launch shapes: the same bits come out
+        assert torch.equal(t0, t1)
+        ref = oracle_mod.Oracle(shape, w, 1, 2, mlp_tokens=1).encode_full(f0)
+        assert_tokens_close(t1.float().cpu().numpy(), ref, "identical frames")
+        assert enc.device_status() == 0
+    finally:
+        enc.close()

@@ -106,3 +106,11 @@ def test_so400m_1view_prefix_key_scores(pkg, oracle_mod):
     stats = run_side_by_side(pkg, oracle_mod, wl.shape, w, _frames(wl, 3),
                              score_source=synth.SCORE_KEY0)
     assert all(0 < s[2][0] < wl.shape.n_tokens for s in stats[1:])
+
+
+def test_so400m_1view_prefix_mlp_all_tokens(pkg, oracle_mod):
+    wl = synth.WORKLOADS["so400m_224_1view"]
+    w = synth.make_weights(wl.shape, 0)
+    stats = run_side_by_side(pkg, oracle_mod, wl.shape, w, _frames(wl, 3), check_caches=True,
+                             mlp_tokens=1)
+    assert all(0 < s[2][0] < wl.shape.n_tokens for s in stats[1:])
