@@ -275,10 +275,10 @@ def main() -> None:
 
     step_ms = {}
 
-    def timed(fn_step, label):
+    def timed(fn_step, label, encoder=None):
         """Full encode of frame 0, warm-up frames, then K timed steps (CUDA events on the
         launch stream, one after every step for the per-step distribution)."""
-        enc.encode_full(frames_dev[0], out)
+        (encoder or enc).encode_full(frames_dev[0], out)
         for t in range(args.warmup):
             fn_step(1 + t)
         barrier()
@@ -336,6 +336,33 @@ def main() -> None:
     pkg.ivit_profile_enable(enc.h, False)
     status = enc.device_status()
 
+    # Approximation quality (a diagnostic, not gated): per-token cosine between the
+    # incremental output and a full re-encode of the same frame, over a few frames.
+    ref_enc = pkg.IncrementalViT.for_workload(wl, weights)
+
+    def quality(encoder, n=8):
+        n = min(n, n_frames - 1)
+        encoder.encode_full(frames_dev[0], out)
+        means, low = [], 1.0
+        for t in range(1, 1 + n):
+            a, _ = encoder.encode_incremental(frames_dev[t])
+            b = ref_enc.encode_full(frames_dev[t])
+            c = torch.nn.functional.cosine_similarity(a.float(), b.float(), dim=-1)
+            means.append(float(c.mean()))
+            low = min(low, float(c.min()))
+        return {"frames": n, "mean_token_cosine": float(np.mean(means)), "min_token_cosine": low}
+
+    quality_default = quality(enc)
+    # The other reading of Sec. III-B: attention on the updated tokens, MLP on every token.
+    import dataclasses
+    enc_all = pkg.IncrementalViT.for_workload(dataclasses.replace(wl, mlp_tokens=1), weights)
+    all_ms = timed(lambda t: pkg.ivit_encode_incremental(enc_all.h, frames_dev[t], out, counts[t], stream),
+                   "mlp_all_tokens", enc_all)
+    mlp_all = {"ms_per_step": all_ms / args.steps, "speedup_vs_full": full_ms / all_ms,
+               "quality_vs_full": quality(enc_all), "device_status": enc_all.device_status()}
+    enc_all.close()
+    ref_enc.close()
+
     frames_total = args.steps * wl.sv * world
     value = frames_total / (inc_ms / 1e3)
     achieved = (gemm_bytes / gemm_n) / (gemm_ms / gemm_n / 1e3) / 1e9 if gemm_n else None
@@ -359,6 +386,8 @@ def main() -> None:
         "full_encode_frames_per_s": frames_total / (full_ms / 1e3),
         "speedup_vs_full": full_ms / inc_ms,
         "odd_even_ms_per_step": 0.5 * (full_ms + inc_ms) / args.steps,  # Sec. III-B chunking
+        "quality_vs_full": quality_default,
+        "mlp_all_tokens": mlp_all,
         "e2e": {"value": frames_total / (e2e_ms / 1e3), "unit": "frames/s",
                 "ms_per_step": e2e_ms / args.steps,
                 "h2d_bytes_per_step": int(frames[0].nbytes),
