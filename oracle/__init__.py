@@ -78,6 +78,8 @@ def lib() -> C.CDLL:
         L.orc_attention.argtypes = [P, C.c_int, P, P, C.c_int, C.c_int, C.c_int, C.c_int,
                                     P, C.c_int]
         L.orc_layer0_keys.argtypes = [P, P, P, P, P, P, C.c_int, C.c_int, C.c_float, P]
+        L.orc_action_combine.argtypes = [P, P, P, P, P, P, C.c_int, C.c_int, P]
+        L.orc_euler.argtypes = [P, P, C.c_int, C.c_float, C.c_int, C.c_int, P]
         _lib = L
     return _lib
 
@@ -235,3 +237,23 @@ def attention(q, k, v) -> np.ndarray:
     o = np.empty((m, dh), np.float32)
     lib().orc_attention(_p(q), dh, _p(k), _p(v), dh, m, n, dh, _p(o), dh)
     return o
+
+
+def action_combine(x0, v0, v7, alpha, beta, b=None) -> np.ndarray:
+    """Eq. 9: x_T = x_0 + alpha v_0 + beta v_7 + b; x0, v0, v7, b [B, A], alpha, beta [B]."""
+    x0, v0, v7, al, be = (_f32(a) for a in (x0, v0, v7, alpha, beta))
+    bb = _f32(b) if b is not None else None
+    B, A = x0.shape
+    out = np.empty((B, A), np.float32)
+    lib().orc_action_combine(_p(x0), _p(v0), _p(v7), _p(al), _p(be), _p(bb) if bb is not None else None,
+                             B, A, _p(out))
+    return out
+
+
+def euler(x0, v, dt: float) -> np.ndarray:
+    """x_T = x_0 + sum_t dt v_t; x0 [B, A], v [T, B, A]."""
+    x0, v = _f32(x0), _f32(v)
+    B, A = x0.shape
+    out = np.empty((B, A), np.float32)
+    lib().orc_euler(_p(x0), _p(v), v.shape[0], float(dt), B, A, _p(out))
+    return out

@@ -582,3 +582,25 @@ int orc_get_cache(const orc_state* s, int which, int layer, float* out) {
   memcpy(out, src, sizeof(float) * view);
   return 0;
 }
+
+/* Eq. 9: the final action state from the two anchor velocities. */
+void orc_action_combine(const float* x0, const float* v0, const float* v7, const float* alpha,
+                        const float* beta, const float* b, int batch, int dim, float* xT) {
+  for (int s = 0; s < batch; ++s)
+    for (int i = 0; i < dim; ++i) {
+      const size_t k = (size_t)s * dim + i;
+      const double y = (double)x0[k] + (double)alpha[s] * v0[k] + (double)beta[s] * v7[k] +
+                       (b ? (double)b[k] : 0.0);
+      xT[k] = (float)y;
+    }
+}
+
+/* Euler integration of the velocity sequence (the sum Eq. 9 compresses). */
+void orc_euler(const float* x0, const float* v, int steps, float dt, int batch, int dim, float* xT) {
+  const size_t n = (size_t)batch * dim;
+  for (size_t k = 0; k < n; ++k) {
+    double y = x0[k];
+    for (int t = 0; t < steps; ++t) y += (double)dt * v[(size_t)t * n + k];
+    xT[k] = (float)y;
+  }
+}

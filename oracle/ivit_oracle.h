@@ -101,6 +101,16 @@ void orc_layer0_keys(const float* e, const float* pos, const float* ln_g, const 
 void orc_attention(const float* q, int q_stride, const float* k, const float* v,
                    int kv_stride, int m, int n, int dh, float* o, int o_stride);
 
+/* ---- the 2-step action combine (Sec. III-C, Eq. 9), for B samples of A action values ---- */
+
+/* x_T[s][i] = x_0[s][i] + alpha[s] v_0[s][i] + beta[s] v_7[s][i] + b[s][i] (b may be NULL:
+ * zero).  The anchor velocities v_0, v_7 and the coefficients come from the caller. */
+void orc_action_combine(const float* x0, const float* v0, const float* v7, const float* alpha,
+                        const float* beta, const float* b, int batch, int dim, float* xT);
+/* Euler integration the combine approximates (the equation before Eq. 9):
+ * x_T = x_0 + sum_t dt v_t over T steps; v [T][B][A]. */
+void orc_euler(const float* x0, const float* v, int steps, float dt, int batch, int dim, float* xT);
+
 #ifdef __cplusplus
 }
 #endif
