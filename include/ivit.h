@@ -189,6 +189,18 @@ int ivit_select_noalloc(const float* e_cur_dev, const float* e_ref_dev, int32_t 
                         int32_t topk, int32_t* idx_out_dev, int32_t* counts_out_dev,
                         void* stream);
 
+/* The 2-step action combine of the flow-matching head (Sec. III-C, Eq. 9):
+ *   xT[s][i] = x0[s][i] + alpha[s] v0[s][i] + beta[s] v7[s][i] + b[s][i]
+ * for `batch` samples of `dim` action values (row-major [batch][dim], fp32, device
+ * memory; alpha, beta fp32 [batch]; b may be NULL, read as zero).  v0 and v7 are the
+ * solver's anchor velocities (first and eighth step) and (alpha, beta, b) the adaptor's
+ * prediction, all computed by the caller: this library holds neither network.  Needs no
+ * handle; enqueued on `stream`, no allocation.  IVIT_ERR_ARG for negative sizes or a
+ * NULL required pointer; batch * dim == 0 does nothing. */
+int ivit_action_combine(const float* x0_dev, const float* v0_dev, const float* v7_dev,
+                        const float* alpha_dev, const float* beta_dev, const float* b_dev,
+                        int32_t batch, int32_t dim, float* xT_dev, void* stream);
+
 /* Message of the last failure on `h` (or of the last failed create if h is NULL). */
 const char* ivit_last_error(const ivit_handle* h);
 

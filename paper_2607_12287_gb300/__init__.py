@@ -29,7 +29,7 @@ EXPORTED = [
     "ivit_weights_size", "ivit_create", "ivit_encode_full", "ivit_encode_incremental",
     "ivit_get_changed", "ivit_get_cache", "ivit_reset", "ivit_profile_enable",
     "ivit_profile_read", "ivit_device_status", "ivit_last_launch_count", "ivit_destroy",
-    "ivit_last_error", "ivit_select_noalloc",
+    "ivit_last_error", "ivit_select_noalloc", "ivit_action_combine",
 ]
 IVIT_NOALLOC_MAX_TOKENS = 65536
 
@@ -81,6 +81,7 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.ivit_destroy.restype = None
     L.ivit_last_error.restype = C.c_char_p
     L.ivit_last_error.argtypes = [P]
+    L.ivit_action_combine.argtypes = [P, P, P, P, P, P, C.c_int32, C.c_int32, P, P]
     L.ivit_select_noalloc.argtypes = [P, P, C.c_int32, C.c_int32, C.c_int32, C.c_int32,
                                       C.c_float, C.c_int32, P, P, P]
     _lib = L
@@ -188,6 +189,15 @@ def ivit_select_noalloc(e_cur, e_ref, n_views: int, n_tok: int, dim: int, select
     that cannot allocate, e.g. while a stream is being captured into a CUDA graph."""
     _check(load().ivit_select_noalloc(_ptr(e_cur), _ptr(e_ref), n_views, n_tok, dim, select_mode,
                                       threshold, topk, _ptr(idx_out), _ptr(counts_out),
+                                      _stream(stream)), None)
+
+
+def ivit_action_combine(x0, v0, v7, alpha, beta, b, xT, stream=None) -> None:
+    """Eq. 9 action combine on device tensors: x0, v0, v7, b (or None), xT fp32 [B, A];
+    alpha, beta fp32 [B]."""
+    B, A = (int(x0.shape[0]), int(x0.shape[1])) if x0.dim() == 2 else (0, 0)
+    _check(load().ivit_action_combine(_ptr(x0), _ptr(v0), _ptr(v7), _ptr(alpha), _ptr(beta),
+                                      _ptr(b) if b is not None else None, B, A, _ptr(xT),
                                       _stream(stream)), None)
 
 
