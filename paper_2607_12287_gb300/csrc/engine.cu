@@ -120,6 +120,7 @@ struct ivit_handle {
   float *e_t = nullptr, *e_ref = nullptr, *sims = nullptr, *x = nullptr;
   float* key_t = nullptr;          // first-layer keys of every token (score_source KEY0)
   float* acache = nullptr;         // [L][M_max][D] attention-block outputs (mlp_tokens ALL)
+  float* gemm_partials = nullptr;  // split-K exchange slots of the GEMMs (global scratch)
   int* rowtok_all = nullptr;       // identity row -> token map, all SV*N rows
   int* m_all = nullptr;            // device copy of SV*N
   CUtensorMap tm_wk0;              // layer 0's key projection (rows D..2D-1 of W_qkv)
@@ -487,6 +488,12 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   const size_t o_err = sa.take(4);
   const size_t o_key = c.score_source == IVIT_SCORE_KEY0 ? sa.take(M * D * 4) : 0;
   const size_t o_acache = c.mlp_tokens == IVIT_MLP_ALL ? sa.take(L * M * D * 4) : 0;
+  // slots for every plan: clusters x CTAs per cluster x row tile x 128 features, fp32
+  size_t part_floats = 0;
+  for (int g = 0; g < kGemmSlots; ++g)
+    for (const GemmPlan* pl : {&h->plan_full[g], &h->plan_inc[g]})
+      part_floats = std::max(part_floats, static_cast<size_t>(pl->n_clusters) * pl->csize * pl->bn * 128);
+  const size_t o_gpart = sa.take(part_floats * 4);
   const size_t o_rta = sa.take(M * 4), o_mall = sa.take(4);
   const size_t o_fb = sa.take(static_cast<size_t>(h->SV) * c.img_h * c.img_w * 3);
   const size_t o_cb = sa.take(h->SV * 4);
@@ -513,6 +520,7 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   h->err = sa.at<int>(o_err);
   if (c.score_source == IVIT_SCORE_KEY0) h->key_t = sa.at<float>(o_key);
   if (c.mlp_tokens == IVIT_MLP_ALL) h->acache = sa.at<float>(o_acache);
+  h->gemm_partials = sa.at<float>(o_gpart);
   h->rowtok_all = sa.at<int>(o_rta);
   h->m_all = sa.at<int>(o_mall);
   {
@@ -575,6 +583,7 @@ double gemm_bytes(int n_out, int k, int kind, long long M) {
 int gemm(ivit_handle* h, const GemmPlan& plan, const CUtensorMap& tw, const CUtensorMap& tx,
          ivit::GemmArgs a, cudaStream_t s) {
   a.err = h->err;
+  a.partials = h->gemm_partials;
   EventPair* ev = nullptr;
   if (h->profiling) {
     if (h->prof_used == h->prof_events.size()) {

@@ -10,9 +10,10 @@
 //
 // The grid is a set of thread-block clusters.  The CTAs of a cluster split K of one
 // output tile between them (so many SMs stream one weight tile at once); each CTA
-// copies its fp32 partial tile from TMEM to its shared memory, and after a cluster
-// barrier every CTA sums a slice of the tile's rows over all CTAs' partials through
-// distributed shared memory, in rank order (deterministic), and runs the epilogue.
+// writes its fp32 partial tile from TMEM to its slot of a global scratch (it stays in
+// L2), and after a cluster barrier every CTA sums a slice of the tile's rows over all
+// slots, in rank order (deterministic), and runs the epilogue.  The scratch outlives
+// the CTAs, so a cluster with no further tile leaves without a second barrier.
 // Clusters walk the output tiles (feature tile x row tile) with a stride.
 //
 // Pipeline per CTA (128 threads): warp 0 lane 0 issues TMA loads (weights with an
@@ -129,7 +130,6 @@ __global__ void __launch_bounds__(128, 1)
   const bool has_k = kb1 > kb0;
   const uint64_t pol_w = l2_policy_evict_first();
   const uint64_t pol_x = l2_policy_evict_last();
-  float* part = reinterpret_cast<float*>(smem);  // [rows][BM] fp32 partial (stage area)
 
   // Weights do not depend on earlier kernels: start streaming the first tile's weight
   // stages now, while the previous kernel may still be running.
@@ -240,33 +240,34 @@ __global__ void __launch_bounds__(128, 1)
         }
       }
     } else {
-      // Partials stay in each CTA's shared memory; every CTA sums a slice of the tile's
-      // rows over all CTAs through distributed shared memory (all loads of a row issued
-      // before the sum), in rank order.
-      if (ok) {
-        if (has_k) {
-          for (int c0 = 0; c0 < rows; c0 += 16) {
-            float v[16];
-            tmem_ld16(trow + c0, v);
+      // Partials go to this CTA's slot of the global scratch (L2); the cluster barrier's
+      // release/acquire makes them visible to the other CTAs, each of which sums a slice
+      // of the tile's rows over all slots in rank order.  Global memory outlives the CTA,
+      // so only a following tile of this cluster (which reuses the slots) needs a second
+      // barrier.
+      float* mine = a.partials + static_cast<size_t>(cl_id * csize + crank) * BN_MAX * BM;
+      if (ok && has_k) {
+        for (int c0 = 0; c0 < rows; c0 += 16) {
+          float v[16];
+          tmem_ld16(trow + c0, v);
 #pragma unroll
-            for (int j = 0; j < 16; ++j)
-              if (c0 + j < rows) part[(c0 + j) * BM + fl] = v[j];
-          }
-        } else {
-          for (int c = 0; c < rows; ++c) part[c * BM + fl] = 0.f;
+          for (int j = 0; j < 16; ++j)
+            if (c0 + j < rows) mine[(c0 + j) * BM + fl] = v[j];
         }
+      } else {
+        for (int c = 0; c < rows; ++c) mine[c * BM + fl] = 0.f;
       }
-      cluster_sync();  // every partial of this tile is in its CTA's shared memory
+      cluster_sync();  // every partial of this tile is in the scratch
       if (ok) {
         const int c_lo = crank * rows / csize, c_hi = (crank + 1) * rows / csize;
         const int f4 = ft * BM + 4 * lane;
-        const uint32_t part_addr = smem_u32(part);
+        const float* slots = a.partials + static_cast<size_t>(cl_id * csize) * BN_MAX * BM;
         for (int c = c_lo + warp; c < c_hi; c += 4) {
-          const uint32_t off = part_addr + static_cast<uint32_t>((c * BM + 4 * lane) * 4);
           float4 p[MAX_CLUSTER];
 #pragma unroll
           for (int s = 0; s < MAX_CLUSTER; ++s)
-            if (s < csize) p[s] = ld_dsmem_f32x4(mapa_shared(off, s));
+            if (s < csize)
+              p[s] = __ldcg(reinterpret_cast<const float4*>(slots + (static_cast<size_t>(s) * BN_MAX + c) * BM + 4 * lane));
           float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
           for (int s = 0; s < MAX_CLUSTER; ++s)
@@ -282,7 +283,7 @@ __global__ void __launch_bounds__(128, 1)
             if (f4 + j < a.n_out) epilogue_store(a.epi, row0 + c, f4 + j, vals[j]);
         }
       }
-      cluster_sync();  // partials stay valid until every CTA has read them
+      if (tile + n_cl < tiles) cluster_sync();  // the next tile rewrites the slots
     }
     tc_fence_before();
     __syncthreads();

@@ -74,6 +74,10 @@ struct GemmArgs {
   const int* d_rows = nullptr;   // device row count M (nullptr: use m_static)
   int m_static = 0;
   int* err = nullptr;            // device error word
+  // Split-K exchange scratch (global memory, stays in L2): slot [cluster][rank][BN_MAX][128]
+  // floats for every CTA of the launch.  Required when the launch's clusters have more
+  // than one CTA.
+  float* partials = nullptr;
   GemmEpilogue epi;
 };
 
