@@ -6,7 +6,8 @@
 //
 // Work item = (query tile of up to 128 packed updated rows of view v, head h).  Each
 // item is handled by a thread-block cluster of `ns` CTAs that split the view's keys:
-// CTA rank s takes keys [s*kpc, (s+1)*kpc), kpc = ceil(N / ns) <= 256.  The clusters
+// CTA rank s takes keys [s*kpc, (s+1)*kpc), kpc = ceil(N / ns), in groups of up to 256
+// keys with an online softmax across the groups.  The clusters
 // walk the items with a stride; items past a view's row count (device-resident, written
 // by the selection kernel) are skipped, so one launch shape serves every row count and
 // the launch can sit in a CUDA graph.  Shared memory and TMEM are sized by kpc, so that
@@ -17,13 +18,16 @@
 //   Q tile [128 rows][dh] by TMA (128-byte swizzle, 64-column slices; the padding columns
 //   dh..round16(dh) are zeroed in shared memory); K, V of the CTA's keys by TMA into
 //   [kpc keys][64 columns] slices;
-//   S = Q K^T   tcgen05.mma M = 128, N = the CTA's keys, K = round16(dh), fp32 in TMEM;
-//   softmax     each thread reads its row of S from TMEM; row max m, P = 2^((S - m) c)
+//   per key group (its K/V tile fetched as soon as the previous group's one is consumed):
+//   S = Q K^T   tcgen05.mma M = 128, N = the group's keys, K = round16(dh), fp32 in TMEM;
+//   softmax     each thread reads its row of S from TMEM; running max m, P = 2^((S - m) c)
 //               (c = log2(e) / sqrt(dh)) rounded to bf16 into shared memory as the next
-//               MMA's A operand (K-major, 128-byte swizzle), l = the sum of those values;
-//   O_s = P V   V is the B operand in MN-major form (its rows are the keys = the MMA's
+//               MMA's A operand (K-major, 128-byte swizzle), l = the running sum of those
+//               values;
+//   O_g = P V   V is the B operand in MN-major form (its rows are the keys = the MMA's
 //               K, its columns the head's dims = the MMA's N): one MMA for dims 0..63
-//               and one for the rest, each inside one 64-column swizzle atom;
+//               and one for the rest, each inside one 64-column swizzle atom; the thread
+//               folds O_g into its running output (registers), rescaled when m grows;
 //   merge       every CTA stores the partial (m, l, O_s) of each row into the shared
 //               memory of the row's owner CTA (distributed shared memory stores); after
 //               a cluster barrier the owner combines them in rank order (deterministic):
@@ -47,7 +51,8 @@ constexpr int MAX_SPLITS = 8;
 // 16), identical on host and device.
 struct AttnLayout {
   int nsl;       // 64-column slices per row
-  int kpad;      // keys per CTA rounded up to 64 (K/V slice rows)
+  int kgrp;      // keys per group: the CTA's keys, at most AKMAX (more run in several groups)
+  int kpad;      // keys per group rounded up to 64 (K/V slice rows)
   int kslice;    // bytes of one K or V slice
   int rp, pst;   // merge: row slots per owner, row stride of a partial output (floats)
   int off_q, off_p, off_k, off_v, off_part, off_bar, bytes;
@@ -57,7 +62,8 @@ struct AttnLayout {
 __host__ __device__ inline AttnLayout attn_layout(int kpc, int dhp, int ns) {
   AttnLayout L;
   L.nsl = dhp > 64 ? 2 : 1;
-  L.kpad = (kpc + 63) / 64 * 64;
+  L.kgrp = kpc < AKMAX ? kpc : AKMAX;
+  L.kpad = (L.kgrp + 63) / 64 * 64;
   L.kslice = L.kpad * 128;
   L.rp = (AQ + ns - 1) / ns;
   L.pst = dhp + 4;
@@ -119,8 +125,10 @@ __global__ void __launch_bounds__(128, 1)
   const int ns = static_cast<int>(cluster_nctarank()), rank = static_cast<int>(cluster_ctarank());
   const int cl = blockIdx.x / ns, ncl = gridDim.x / ns;
   const int kpc = (N + ns - 1) / ns;
-  const int k0 = rank * kpc, nk = max(0, min(kpc, N - k0)), nks = (nk + 15) & ~15;
+  const int k0 = rank * kpc, nk = max(0, min(kpc, N - k0));  // this CTA's keys
   const AttnLayout L = attn_layout(kpc, DHP, ns);
+  const int G = L.kgrp;                                      // keys per group
+  const int ngroups = (nk + G - 1) / G;
   const int NSL = L.nsl;
   const uint32_t sb = smem_u32(sm);
   const uint32_t bq = sb + L.off_bar, bk = bq + 8, bv = bq + 16, bs = bq + 24, bo = bq + 32;
@@ -161,43 +169,47 @@ __global__ void __launch_bounds__(128, 1)
   const uint32_t tm_s = tmem, tm_o = tmem + static_cast<uint32_t>(L.tm_o);
   const uint64_t pol_q = l2_policy_evict_first(), pol_kv = l2_policy_evict_last();
 
-  // K or V of this CTA's keys of item (v, h): boxes of 64 keys x 64 dims per slice.
-  auto load_kv = [&](uint32_t bar, int off, const CUtensorMap* map, int v, int h) {
-    const int nbox = (nk + KROWS - 1) / KROWS;
+  // K or V of key group g of this CTA's keys of item (v, h): boxes of 64 keys x 64 dims
+  // per slice.
+  auto load_kv = [&](uint32_t bar, int off, const CUtensorMap* map, int v, int h, int g) {
+    const int gk0 = k0 + g * G, gn = min(G, nk - g * G);
+    const int nbox = (gn + KROWS - 1) / KROWS;
     mbar_arrive_expect_tx(bar, static_cast<uint32_t>(nbox * NSL * KROWS * 128));
     for (int sl = 0; sl < NSL; ++sl)
       for (int b = 0; b < nbox; ++b)
-        tma_load_2d(sb + off + sl * L.kslice + b * KROWS * 128, map, h * dh + sl * 64, v * N + k0 + b * KROWS,
+        tma_load_2d(sb + off + sl * L.kslice + b * KROWS * 128, map, h * dh + sl * 64, v * N + gk0 + b * KROWS,
                     bar, pol_kv);
   };
 
-  if (a.prefetch && tid == 0) {
-    load_kv(bk, L.off_k, &tm_k, it.v, it.h);
-    load_kv(bv, L.off_v, &tm_v, it.v, it.h);
+  // Incremental calls whose keys fit one group fetch the cached K/V before the wait.
+  const bool pre = a.prefetch && ngroups == 1;
+  if (pre && tid == 0) {
+    load_kv(bk, L.off_k, &tm_k, it.v, it.h, 0);
+    load_kv(bv, L.off_v, &tm_v, it.v, it.h, 0);
   }
   pdl_wait();  // queries and this call's K/V rows (QKV kernel) are visible from here
   pdl_launch_dependents();
 
-  uint32_t ph = 0;  // completed phases of every barrier (each completes once per item)
+  uint32_t ph_q = 0, ph_g = 0;  // completed phases: bq once per item, the others once per group
   bool ok = true;
   const float sc = rsqrtf(static_cast<float>(dh)) * 1.4426950408889634f;  // log2(e) / sqrt(dh)
   bool first = true;
   while (true) {
-    const bool patch = first && a.prefetch;
+    const bool patch = first && pre;
     first = false;
     if (tid == 0) {
       mbar_arrive_expect_tx(bq, NSL * SLICE_Q);
       for (int sl = 0; sl < NSL; ++sl)
         tma_load_2d(sb + L.off_q + sl * SLICE_Q, &tm_q, it.h * dh + sl * 64, it.r0, bq, pol_q);
-      if (!patch) {
-        load_kv(bk, L.off_k, &tm_k, it.v, it.h);
-        load_kv(bv, L.off_v, &tm_v, it.v, it.h);
+      if (!patch && ngroups > 0) {
+        load_kv(bk, L.off_k, &tm_k, it.v, it.h, 0);
+        load_kv(bv, L.off_v, &tm_v, it.v, it.h, 0);
       }
     }
     if (patch) {
       // the prefetched tiles hold the cache as it was before the QKV kernel: overwrite
       // the rows of the tokens it updated that fall in this CTA's key range
-      if (!mbar_wait(bk, ph & 1) || !mbar_wait(bv, ph & 1)) ok = false;
+      if (!mbar_wait(bk, ph_g & 1) || !mbar_wait(bv, ph_g & 1)) ok = false;
       const int rb = a.cu_rows[it.v], m = a.cu_rows[it.v + 1] - rb;
       const int dh8 = dh >> 3;
       for (int e = tid; e < m * dh8; e += blockDim.x) {
@@ -210,7 +222,8 @@ __global__ void __launch_bounds__(128, 1)
         *reinterpret_cast<uint4*>(sm + L.off_v + off) = __ldcg(reinterpret_cast<const uint4*>(a.cache_v + g));
       }
     }
-    if (!mbar_wait(bq, ph & 1)) ok = false;
+    if (!mbar_wait(bq, ph_q & 1)) ok = false;
+    ++ph_q;
     if (DHP != dh) {  // columns dh..dh+7 of the Q tile hold the next head: zero them
       const int c = dh >> 3;
       *reinterpret_cast<uint4*>(sm + L.off_q + (c >> 3) * SLICE_Q + swz(tid, c & 7)) = make_uint4(0, 0, 0, 0);
@@ -219,93 +232,117 @@ __global__ void __launch_bounds__(128, 1)
     tc_fence_before();
     __syncthreads();
 
-    // ---- S = Q K^T
-    if (tid == 0) {
-      tc_fence_after();
-      if (!mbar_wait(bk, ph & 1)) ok = false;
-      tc_fence_after();
-      if (ok && nk > 0) {
-        const uint32_t id = idesc_bf16_f32(AQ, nks);
-#pragma unroll
-        for (int t = 0; t < DHP / 16; ++t) {
-          const uint32_t qo = sb + L.off_q + (t >> 2) * SLICE_Q + (t & 3) * 32;
-          const uint32_t ko = sb + L.off_k + (t >> 2) * L.kslice + (t & 3) * 32;
-          umma_bf16(tm_s, sdesc_kmajor_sw128(qo), sdesc_kmajor_sw128(ko), id, t > 0);
-        }
-      }
-      umma_commit(bs);
-    }
-    __syncwarp();
-    if (!mbar_wait(bs, ph & 1)) ok = false;
-    tc_fence_after();
-
-    // ---- softmax over this CTA's keys, P to shared memory
-    const bool wact = warp * 32 < it.nq && nk > 0;  // warp-uniform; padding warps skip the math
+    // Online softmax over the key groups (running max m, running sum l, output in
+    // registers rescaled by 2^((m_old - m_new) c) when the max grows).
+    const bool wrow = warp * 32 < it.nq;  // warp-uniform: padding warps skip the math
     float m_run = -INFINITY, l_run = 0.f;
-    if (wact) {
-      for (int cb = 0; cb < nks; cb += 64) {
-        uint32_t r0[32], r1[32];
-        tmem_ld32_async(trow + cb, r0);
-        tmem_ld32_async(trow + cb + 32, r1);
-        tmem_ld_wait();
+    float o_run[DHP];
 #pragma unroll
-        for (int u = 0; u < 32; ++u) {
-          if (cb + u < nk) m_run = fmaxf(m_run, __uint_as_float(r0[u]));
-          if (cb + 32 + u < nk) m_run = fmaxf(m_run, __uint_as_float(r1[u]));
+    for (int d = 0; d < DHP; ++d) o_run[d] = 0.f;
+    for (int g = 0; g < ngroups; ++g) {
+      const int gn = min(G, nk - g * G), gns = (gn + 15) & ~15;
+      // ---- S = Q K^T
+      if (tid == 0) {
+        tc_fence_after();
+        if (!mbar_wait(bk, ph_g & 1)) ok = false;
+        tc_fence_after();
+        if (ok) {
+          const uint32_t id = idesc_bf16_f32(AQ, gns);
+#pragma unroll
+          for (int t = 0; t < DHP / 16; ++t) {
+            const uint32_t qo = sb + L.off_q + (t >> 2) * SLICE_Q + (t & 3) * 32;
+            const uint32_t ko = sb + L.off_k + (t >> 2) * L.kslice + (t & 3) * 32;
+            umma_bf16(tm_s, sdesc_kmajor_sw128(qo), sdesc_kmajor_sw128(ko), id, t > 0);
+          }
         }
+        umma_commit(bs);
       }
-      const float mo = m_run * sc;
-      float lsum[4] = {0.f, 0.f, 0.f, 0.f};
-      for (int cb = 0; cb < nks; cb += 32) {
-        uint32_t r[32];
-        tmem_ld32_async(trow + cb, r);
-        tmem_ld_wait();
-        uint32_t pk[16];
-#pragma unroll
-        for (int u = 0; u < 16; ++u) {
-          const int j = cb + 2 * u;
-          const float p0 = j < nk ? ex2(fmaf(__uint_as_float(r[2 * u]), sc, -mo)) : 0.f;
-          const float p1 = j + 1 < nk ? ex2(fmaf(__uint_as_float(r[2 * u + 1]), sc, -mo)) : 0.f;
-          const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
-          const float2 f = __bfloat1622float2(b);
-          lsum[u & 3] += f.x + f.y;  // the normaliser sums the values the MMA multiplies
-          pk[u] = *reinterpret_cast<const uint32_t*>(&b);
-        }
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-          const int kc = (cb >> 3) + q4;  // 16-byte chunk (8 keys) of this row of P
-          if (kc * 8 < nks)
-            *reinterpret_cast<uint4*>(sm + L.off_p + (kc >> 3) * SLICE_Q + swz(tid, kc & 7)) =
-                make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
-        }
-      }
-      l_run = (lsum[0] + lsum[1]) + (lsum[2] + lsum[3]);
-    }
-    fence_proxy_async_shared();
-    tc_fence_before();
-    __syncthreads();
+      __syncwarp();
+      if (!mbar_wait(bs, ph_g & 1)) ok = false;
+      tc_fence_after();
+      if (tid == 0 && g + 1 < ngroups) load_kv(bk, L.off_k, &tm_k, it.v, it.h, g + 1);  // K tile consumed
 
-    // ---- O_s = P V
-    if (tid == 0) {
+      // ---- softmax of the group, P to shared memory
+      float alpha = 1.f;
+      if (wrow) {
+        float mc = -INFINITY;
+        for (int cb = 0; cb < gns; cb += 64) {
+          uint32_t r0[32], r1[32];
+          tmem_ld32_async(trow + cb, r0);
+          tmem_ld32_async(trow + cb + 32, r1);
+          tmem_ld_wait();
+#pragma unroll
+          for (int u = 0; u < 32; ++u) {
+            if (cb + u < gn) mc = fmaxf(mc, __uint_as_float(r0[u]));
+            if (cb + 32 + u < gn) mc = fmaxf(mc, __uint_as_float(r1[u]));
+          }
+        }
+        const float m_new = fmaxf(m_run, mc);
+        alpha = ex2((m_run - m_new) * sc);  // 0 on the first group (m_run = -inf)
+        const float mo = m_new * sc;
+        float lsum[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int cb = 0; cb < gns; cb += 32) {
+          uint32_t r[32];
+          tmem_ld32_async(trow + cb, r);
+          tmem_ld_wait();
+          uint32_t pk[16];
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            const int j = cb + 2 * u;
+            const float p0 = j < gn ? ex2(fmaf(__uint_as_float(r[2 * u]), sc, -mo)) : 0.f;
+            const float p1 = j + 1 < gn ? ex2(fmaf(__uint_as_float(r[2 * u + 1]), sc, -mo)) : 0.f;
+            const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
+            const float2 f = __bfloat1622float2(b);
+            lsum[u & 3] += f.x + f.y;  // the normaliser sums the values the MMA multiplies
+            pk[u] = *reinterpret_cast<const uint32_t*>(&b);
+          }
+#pragma unroll
+          for (int q4 = 0; q4 < 4; ++q4) {
+            const int kc = (cb >> 3) + q4;  // 16-byte chunk (8 keys) of this row of P
+            if (kc * 8 < gns)
+              *reinterpret_cast<uint4*>(sm + L.off_p + (kc >> 3) * SLICE_Q + swz(tid, kc & 7)) =
+                  make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
+          }
+        }
+        l_run = l_run * alpha + ((lsum[0] + lsum[1]) + (lsum[2] + lsum[3]));
+        m_run = m_new;
+      }
+      fence_proxy_async_shared();
+      tc_fence_before();
+      __syncthreads();
+
+      // ---- O_g = P V, folded into the running output
+      if (tid == 0) {
+        tc_fence_after();
+        if (!mbar_wait(bv, ph_g & 1)) ok = false;
+        tc_fence_after();
+        if (ok) {
+          const uint32_t id0 = idesc_bf16_f32_bmn(AQ, DHP > 64 ? 64 : DHP);
+          const uint32_t id1 = idesc_bf16_f32_bmn(AQ, DHP > 64 ? DHP - 64 : 16);
+          for (int t = 0; t < gns / 16; ++t) {
+            const uint64_t ad = sdesc_kmajor_sw128(sb + L.off_p + (t >> 2) * SLICE_Q + (t & 3) * 32);
+            umma_bf16(tm_o, ad, sdesc_sw128(sb + L.off_v + t * 2048, 1024, 1024), id0, t > 0);
+            if (DHP > 64)
+              umma_bf16(tm_o + 64, ad, sdesc_sw128(sb + L.off_v + L.kslice + t * 2048, 1024, 1024), id1, t > 0);
+          }
+        }
+        umma_commit(bo);
+      }
+      __syncwarp();
+      if (!mbar_wait(bo, ph_g & 1)) ok = false;
       tc_fence_after();
-      if (!mbar_wait(bv, ph & 1)) ok = false;
-      tc_fence_after();
-      if (ok && nk > 0) {
-        const uint32_t id0 = idesc_bf16_f32_bmn(AQ, DHP > 64 ? 64 : DHP);
-        const uint32_t id1 = idesc_bf16_f32_bmn(AQ, DHP > 64 ? DHP - 64 : 16);
-        for (int t = 0; t < nks / 16; ++t) {
-          const uint64_t ad = sdesc_kmajor_sw128(sb + L.off_p + (t >> 2) * SLICE_Q + (t & 3) * 32);
-          umma_bf16(tm_o, ad, sdesc_sw128(sb + L.off_v + t * 2048, 1024, 1024), id0, t > 0);
-          if (DHP > 64)
-            umma_bf16(tm_o + 64, ad, sdesc_sw128(sb + L.off_v + L.kslice + t * 2048, 1024, 1024), id1, t > 0);
+      ++ph_g;
+      if (tid == 0 && g + 1 < ngroups) load_kv(bv, L.off_v, &tm_v, it.v, it.h, g + 1);  // V tile consumed
+      if (wrow) {  // warp-uniform: tcgen05.ld is a warp-collective instruction
+#pragma unroll
+        for (int c = 0; c < DHP; c += 16) {
+          float ov[16];
+          tmem_ld16(trow + L.tm_o + c, ov);
+#pragma unroll
+          for (int u = 0; u < 16; ++u) o_run[c + u] = o_run[c + u] * alpha + ov[u];
         }
       }
-      umma_commit(bo);
     }
-    __syncwarp();
-    if (!mbar_wait(bo, ph & 1)) ok = false;
-    tc_fence_after();
-    ++ph;
 
     // next item of this cluster (the same for every rank)
     int s_next = s + ncl;
@@ -313,55 +350,36 @@ __global__ void __launch_bounds__(128, 1)
     while (s_next < n_items && !item_at(s_next, a, nxt)) s_next += ncl;
 
     if (ns == 1) {
-      if (wact) {  // warp-uniform: tcgen05.ld is a warp-collective instruction
+      if (wrow && tid < it.nq) {
         const float inv = 1.f / l_run;
         bf16* orow = a.o + static_cast<size_t>(it.r0 + tid) * D + it.h * dh;
 #pragma unroll
-        for (int c = 0; c < DHP; c += 16) {
-          float ov[16];
-          tmem_ld16(trow + L.tm_o + c, ov);
+        for (int c = 0; c < DHP; c += 8) {
+          if (c < dh) {
+            uint4 u;
+            uint32_t* w = reinterpret_cast<uint32_t*>(&u);
 #pragma unroll
-          for (int h8 = 0; h8 < 16; h8 += 8) {
-            if (tid < it.nq && c + h8 < dh) {
-              uint4 u;
-              uint32_t* w = reinterpret_cast<uint32_t*>(&u);
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const __nv_bfloat162 b =
-                    __floats2bfloat162_rn(ov[h8 + 2 * e] * inv, ov[h8 + 2 * e + 1] * inv);
-                w[e] = *reinterpret_cast<const uint32_t*>(&b);
-              }
-              *reinterpret_cast<uint4*>(orow + c + h8) = u;
+            for (int e = 0; e < 4; ++e) {
+              const __nv_bfloat162 b = __floats2bfloat162_rn(o_run[c + 2 * e] * inv, o_run[c + 2 * e + 1] * inv);
+              w[e] = *reinterpret_cast<const uint32_t*>(&b);
             }
+            *reinterpret_cast<uint4*>(orow + c) = u;
           }
         }
       }
     } else {
       // push this CTA's partial (m, l, O_s) of row i to slot [rank][i - owner * rpi] of
-      // the owner CTA i / rpi; key-less CTAs push a neutral partial (m = -inf, l = 0)
+      // the owner CTA i / rpi; a CTA without keys pushes m = -inf, l = 0, O = 0
       const int rpi = (it.nq + ns - 1) / ns;  // rows per owner in this item (<= rp)
-      const bool mine = tid < it.nq;
-      const int owner = mine ? tid / rpi : 0, slot = tid - owner * rpi;
-      const uint32_t obase = mapa_shared(smem_u32(po + (rank * L.rp + slot) * L.pst), static_cast<uint32_t>(owner));
-      if (warp * 32 < it.nq) {  // warp-uniform
-        if (wact) {
+      if (tid < it.nq) {
+        const int owner = tid / rpi, slot = tid - owner * rpi;
+        const uint32_t obase =
+            mapa_shared(smem_u32(po + (rank * L.rp + slot) * L.pst), static_cast<uint32_t>(owner));
 #pragma unroll
-          for (int c = 0; c < DHP; c += 16) {
-            float ov[16];
-            tmem_ld16(trow + L.tm_o + c, ov);
-            if (mine)
-#pragma unroll
-              for (int q = 0; q < 16; q += 4)
-                st_dsmem_f32x4(obase + 4 * (c + q), make_float4(ov[q], ov[q + 1], ov[q + 2], ov[q + 3]));
-          }
-        } else if (mine) {
-#pragma unroll
-          for (int c = 0; c < DHP; c += 4) st_dsmem_f32x4(obase + 4 * c, make_float4(0.f, 0.f, 0.f, 0.f));
-        }
-        if (mine) {
-          st_dsmem_f32(mapa_shared(smem_u32(pm + rank * L.rp + slot), static_cast<uint32_t>(owner)), m_run);
-          st_dsmem_f32(mapa_shared(smem_u32(pl + rank * L.rp + slot), static_cast<uint32_t>(owner)), l_run);
-        }
+        for (int c = 0; c < DHP; c += 4)
+          st_dsmem_f32x4(obase + 4 * c, make_float4(o_run[c], o_run[c + 1], o_run[c + 2], o_run[c + 3]));
+        st_dsmem_f32(mapa_shared(smem_u32(pm + rank * L.rp + slot), static_cast<uint32_t>(owner)), m_run);
+        st_dsmem_f32(mapa_shared(smem_u32(pl + rank * L.rp + slot), static_cast<uint32_t>(owner)), l_run);
       }
       cluster_sync();  // every rank's partials of this CTA's rows are in its shared memory
       const int lo = rank * rpi, nmine = max(0, min(it.nq, lo + rpi) - lo);
@@ -463,7 +481,7 @@ cudaError_t attention_tc_setup() {
 cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
                                 const AttnTcArgs& a, int max_ctas, cudaStream_t s) {
   const int ns = a.key_splits;
-  if (ns < 1 || ns > MAX_SPLITS || (a.n_tok + ns - 1) / ns > AKMAX) return cudaErrorInvalidValue;
+  if (ns < 1 || ns > MAX_SPLITS) return cudaErrorInvalidValue;
   const int items = a.sv * a.heads * a.qtiles;
   const int clusters = max(1, min(items, max_ctas / ns));
   const int grid = clusters * ns;

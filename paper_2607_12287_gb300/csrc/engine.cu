@@ -348,18 +348,17 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   IVIT_CK(h, ivit::attention_tc_setup());
   if (const char* at = std::getenv("IVIT_ATTN")) h->attn_tc = std::string(at) != "simt";
   {
-    // Key splits of the tensor-core attention: at most 128 keys per CTA (when 8 splits
-    // allow it), at least 64; within that, as many as fill the SMs once for the expected
-    // items (query tiles x heads x views: all tokens when full, a tenth when incremental),
-    // then more while one CTA's shared memory exceeds the device limit.
+    // Key splits of the tensor-core attention: as many as fill the SMs once for the
+    // expected items (query tiles x heads x views: all tokens when full, a tenth when
+    // incremental), at least 64 keys per CTA, one (online softmax over key groups) when
+    // the items alone fill the GPU; more while one CTA's shared memory exceeds the limit.
     int optin = 0;
     IVIT_CK(h, cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device));
     const int dh = h->D / h->H;
     auto splits = [&](int m_exp) {
-      const int ns_min = std::min(8, std::max((h->N + 255) / 256, (h->N + 127) / 128));
-      const int ns_cap = std::max(ns_min, std::min(8, (h->N + 63) / 64));
+      const int ns_cap = std::max(1, std::min(8, (h->N + 63) / 64));  // at least 64 keys per CTA
       const int items = h->SV * h->H * ((m_exp + 127) / 128);
-      int ns = std::max(ns_min, std::min(ns_cap, h->num_sms / std::max(1, items)));
+      int ns = std::max(1, std::min(ns_cap, h->num_sms / std::max(1, items)));
       while (ns < 8 && ivit::attention_tc_smem(h->N, dh, ns) > static_cast<size_t>(optin)) ++ns;
       return ns;
     };

@@ -224,3 +224,12 @@ def test_mlp_all_tokens_identical_frames(pkg, oracle_mod):
         assert enc.device_status() == 0
     finally:
         enc.close()
+
+
+def test_many_keys_online_softmax_groups(pkg, oracle_mod):
+    # N = 324 keys per view and 32 views: the full encode has enough items to run one CTA
+    # per item, which walks the keys in two groups (256 + 68) with the online softmax
+    shape = synth.EncoderShape(288, 288, 16, 128, 2, 2, 256, synth.GELU_TANH)
+    w = synth.make_weights(shape, 131)
+    frames = list(synth.stream_random(shape, 32, 3, 132, change_p=0.15))
+    run_side_by_side(pkg, oracle_mod, shape, w, frames, 16, 2, check_caches=True)
