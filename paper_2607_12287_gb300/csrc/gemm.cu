@@ -41,10 +41,18 @@ struct GemmSmem {
   static constexpr int TOTAL = BAR_OFFSET + 256 + 1024;  // barriers, flags, 1 KB alignment slack
 };
 
+// Hardware tanh (one MUFU instruction, relative error about 2^-11: below the bf16
+// rounding the GELU output gets).
+__device__ __forceinline__ float tanh_hw(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ float gelu_f(float x, int mode) {
   if (mode == 1) return 0.5f * x * (1.f + erff(x * 0.70710678118654752f));
   const float c = 0.79788456080286536f;  // sqrt(2/pi)
-  return 0.5f * x * (1.f + tanhf(c * (x + 0.044715f * x * x * x)));
+  return 0.5f * x * (1.f + tanh_hw(c * (x + 0.044715f * x * x * x)));
 }
 
 __device__ __forceinline__ void epilogue_store(const GemmEpilogue& e, int r, int f, float y) {
@@ -296,9 +304,187 @@ __global__ void __launch_bounds__(128, 1)
   }
 }
 
+// Many-tile form for single-CTA clusters (large row counts): a persistent loop over the
+// tiles with warp specialisation, so the epilogue of one tile overlaps the main loop of
+// the next.  Warps 0-3 drain the accumulator (TMEM lane = output feature), warp 4 lane
+// 0 issues the TMA loads, warp 5 lane 0 issues the MMAs; two TMEM accumulators
+// (acc_full: MMAs done -> epilogue, acc_empty: epilogue done -> MMAs).
+constexpr int WS_THREADS = 192;
+
+template <int BN_MAX>
+__global__ void __launch_bounds__(WS_THREADS, 1)
+    gemm_ws_kernel(const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_x,
+                   const GemmArgs a) {
+  using L = GemmSmem<BN_MAX>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR_OFFSET);
+  // full[STAGES], empty[STAGES], acc_full[2], acc_empty[2], TMEM slot, abort flag
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 4);
+  volatile int* sh_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t smem_base = smem_u32(smem), bar_base = smem_u32(bars);
+  const uint32_t accf = bar_base + 8 * (2 * STAGES), acce = accf + 16;
+
+  if (tid == 0) {
+    for (int st = 0; st < STAGES; ++st) {
+      mbar_init(bar_base + 8 * st, 1);
+      mbar_init(bar_base + 8 * (STAGES + st), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(accf + 8 * b, 1);
+      mbar_init(acce + 8 * b, 4);  // one arrival per epilogue warp
+    }
+    fence_mbar_init();
+    tma_prefetch_desc(&tm_w);
+    tma_prefetch_desc(&tm_x);
+    *sh_abort = 0;
+  }
+  if (warp == 5) {
+    tmem_alloc(smem_u32(tmem_slot), 2 * BN_MAX);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  const int M = a.d_rows ? *a.d_rows : a.m_static;
+  const int n_ft = (a.n_out + BM - 1) / BM;
+  const int n_tt = (M + BN_MAX - 1) / BN_MAX;
+  const int n_kb = (a.k + BK - 1) / BK;
+  const int tiles = n_ft * n_tt;
+
+  // first tile's weight stages before the programmatic-launch wait (constants)
+  // (the row count is from the selection kernel, at least two launches back)
+  int n_pre = 0;
+  if (warp == 4 && lane == 0 && static_cast<int>(blockIdx.x) < tiles) {
+    const int ft = blockIdx.x % n_ft, tt = blockIdx.x / n_ft;
+    const int rows = min(BN_MAX, M - tt * BN_MAX);
+    const int nbox = (((rows + 15) & ~15) + XBOX - 1) / XBOX;
+    n_pre = min(STAGES, n_kb);
+    for (int i = 0; i < n_pre; ++i) {
+      mbar_arrive_expect_tx(bar_base + 8 * i, W_TILE_BYTES + nbox * XBOX_BYTES);  // rows follow after the wait
+      tma_load_2d(smem_base + i * L::STAGE_BYTES, &tm_w, i * BK, ft * BM, bar_base + 8 * i, l2_policy_evict_first());
+    }
+  }
+  pdl_wait();
+  pdl_launch_dependents();
+
+  if (warp == 4) {
+    if (lane == 0) {
+      const uint64_t pol_w = l2_policy_evict_first(), pol_x = l2_policy_evict_last();
+      uint32_t stage = 0, phase = 0;
+      bool first = true;
+      for (int tile = blockIdx.x; tile < tiles && *sh_abort == 0; tile += gridDim.x) {
+        const int ft = tile % n_ft, tt = tile / n_ft;
+        const int row0 = tt * BN_MAX, rows = min(BN_MAX, M - row0);
+        const int nbox = (((rows + 15) & ~15) + XBOX - 1) / XBOX;
+        for (int kb = 0; kb < n_kb; ++kb) {
+          const uint32_t full = bar_base + 8 * stage, empty = bar_base + 8 * (STAGES + stage);
+          const uint32_t st = smem_base + stage * L::STAGE_BYTES;
+          const bool pre = first && kb < n_pre;  // weights already requested, bytes expected
+          if (!pre) {
+            if (!mbar_wait(empty, phase ^ 1)) {
+              atomicExch(a.err, kErrWaitSlotEmpty);
+              *sh_abort = 1;
+              break;
+            }
+            mbar_arrive_expect_tx(full, W_TILE_BYTES + nbox * XBOX_BYTES);
+            tma_load_2d(st, &tm_w, kb * BK, ft * BM, full, pol_w);
+          }
+          for (int b = 0; b < nbox; ++b)
+            tma_load_2d(st + W_TILE_BYTES + b * XBOX_BYTES, &tm_x, kb * BK, row0 + b * XBOX, full, pol_x);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        first = false;
+      }
+    }
+  } else if (warp == 5) {
+    if (lane == 0) {
+      uint32_t stage = 0, phase = 0;
+      int iter = 0;
+      for (int tile = blockIdx.x; tile < tiles && *sh_abort == 0; tile += gridDim.x, ++iter) {
+        const int tt = tile / n_ft;
+        const int rows = min(BN_MAX, M - tt * BN_MAX);
+        const uint32_t idesc = idesc_bf16_f32(BM, (rows + 15) & ~15);
+        const int b = iter & 1;
+        if (!mbar_wait(acce + 8 * b, ((iter >> 1) & 1) ^ 1)) {  // accumulator b drained
+          atomicExch(a.err, kErrWaitAccum);
+          *sh_abort = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t acc = tmem + static_cast<uint32_t>(b * BN_MAX);
+        for (int kb = 0; kb < n_kb; ++kb) {
+          if (!mbar_wait(bar_base + 8 * stage, phase)) {
+            atomicExch(a.err, kErrWaitTmaFull);
+            *sh_abort = 1;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_base + stage * L::STAGE_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k)
+            umma_bf16(acc, sdesc_kmajor_sw128(st + k * 32), sdesc_kmajor_sw128(st + W_TILE_BYTES + k * 32), idesc,
+                      (kb > 0 || k > 0) ? 1u : 0u);
+          umma_commit(bar_base + 8 * (STAGES + stage));
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        umma_commit(accf + 8 * b);  // accumulator b complete
+      }
+    }
+  } else {
+    // epilogue warps 0-3: TMEM lane 32 w + lane = tile-local output feature
+    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    int iter = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++iter) {
+      const int ft = tile % n_ft, tt = tile / n_ft;
+      const int row0 = tt * BN_MAX, rows = min(BN_MAX, M - row0);
+      const int b = iter & 1;
+      if (!mbar_wait(accf + 8 * b, (iter >> 1) & 1)) {
+        atomicExch(a.err, kErrWaitAccum);
+        *sh_abort = 1;
+        break;
+      }
+      tc_fence_after();
+      const int f = ft * BM + warp * 32 + lane;
+      const uint32_t acc = trow + static_cast<uint32_t>(b * BN_MAX);
+      for (int c0 = 0; c0 < rows; c0 += 16) {
+        float v[16];
+        tmem_ld16(acc + c0, v);
+        if (f < a.n_out) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (c0 + j < rows) epilogue_store(a.epi, row0 + c0 + j, f, v[j]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acce + 8 * b);  // accumulator b may be overwritten
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 2 * BN_MAX);
+  }
+}
+
 template <int BN>
 cudaError_t launch_variant(const CUtensorMap& tm_w, const CUtensorMap& tm_x, const GemmArgs& a,
                            int n_clusters, int csize, cudaStream_t s) {
+  if (BN == 256 && csize == 1)
+    return launch_ex(gemm_ws_kernel<BN>, dim3(n_clusters), dim3(WS_THREADS), GemmSmem<BN>::TOTAL, s, 1, tm_w, tm_x,
+                     a);
   // cluster dims are always given (also for a single CTA) so %cluster_nctarank is exact
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(n_clusters * csize);
@@ -343,6 +529,10 @@ cudaError_t setup_variant() {
   cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        GemmSmem<BN>::TOTAL);
   if (e != cudaSuccess) return e;
+  if (BN == 256) {
+    e = cudaFuncSetAttribute(gemm_ws_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmSmem<BN>::TOTAL);
+    if (e != cudaSuccess) return e;
+  }
   return cudaFuncSetAttribute(gemm_tc_kernel<BN>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
 
