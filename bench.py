@@ -228,6 +228,10 @@ def main() -> None:
     ap.add_argument("--impl", default="ivit", choices=["ivit", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu", action="store_true", help="skip the oracle CPU baseline")
+    ap.add_argument("--streams", type=int, default=0,
+                    help="run the workload with this many camera streams (its first ones)")
+    ap.add_argument("--lean", action="store_true",
+                    help="time the incremental and full steps only (one handle: for profiler captures)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -241,6 +245,11 @@ def main() -> None:
         wl = synth.sweep_workload(int(args.workload.rsplit("_", 1)[1].rstrip("pct")) / 100.0)
     else:
         ap.error(f"unknown workload {args.workload}")
+    if args.streams > 0:
+        import dataclasses
+        sv = args.streams * wl.n_views
+        views = wl.views[:sv] if len(wl.views) >= sv else wl.views
+        wl = dataclasses.replace(wl, name=f"{wl.name}_{args.streams}streams", n_streams=args.streams, views=views)
 
     if args.impl == "reference":
         run_reference(args, wl, rank)
@@ -310,6 +319,16 @@ def main() -> None:
     launches_per_step = pkg.ivit_last_launch_count(enc.h)
     changed = counts[1 + args.warmup:].float().sum(1).cpu().numpy()
     full_ms = timed(full_step, "full")
+    if args.lean:  # profiler captures: the two timed passes only
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "lean": True, "config": describe(wl),
+                              "ms_per_step": inc_ms / args.steps, "full_encode_ms_per_step": full_ms / args.steps,
+                              "device_status": enc.device_status(), "clocks": clocks}), flush=True)
+        enc.close()
+        if dist is not None:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
 
     # e2e: host frames (pinned) -> device, encode through the C ABI, tokens + counts -> host
     host_in = [torch.from_numpy(f).pin_memory() for f in frames]
