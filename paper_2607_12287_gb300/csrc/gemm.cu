@@ -306,10 +306,12 @@ __global__ void __launch_bounds__(128, 1)
 
 // Many-tile form for single-CTA clusters (large row counts): a persistent loop over the
 // tiles with warp specialisation, so the epilogue of one tile overlaps the main loop of
-// the next.  Warps 0-3 drain the accumulator (TMEM lane = output feature), warp 4 lane
-// 0 issues the TMA loads, warp 5 lane 0 issues the MMAs; two TMEM accumulators
-// (acc_full: MMAs done -> epilogue, acc_empty: epilogue done -> MMAs).
-constexpr int WS_THREADS = 192;
+// the next.  Warps 0-7 drain the accumulator (warp w reads TMEM lane quarter w % 4 =
+// 32 output features, rows of half w / 4 of the tile), warp 8 lane 0 issues the TMA
+// loads, warp 9 lane 0 issues the MMAs; two TMEM accumulators (acc_full: MMAs done ->
+// epilogue, acc_empty: all eight epilogue warps done -> MMAs).
+constexpr int WS_EPI_WARPS = 8;
+constexpr int WS_THREADS = (WS_EPI_WARPS + 2) * 32;
 
 template <int BN_MAX>
 __global__ void __launch_bounds__(WS_THREADS, 1)
@@ -334,14 +336,14 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(accf + 8 * b, 1);
-      mbar_init(acce + 8 * b, 4);  // one arrival per epilogue warp
+      mbar_init(acce + 8 * b, WS_EPI_WARPS);  // one arrival per epilogue warp
     }
     fence_mbar_init();
     tma_prefetch_desc(&tm_w);
     tma_prefetch_desc(&tm_x);
     *sh_abort = 0;
   }
-  if (warp == 5) {
+  if (warp == WS_EPI_WARPS + 1) {
     tmem_alloc(smem_u32(tmem_slot), 2 * BN_MAX);
     tmem_relinquish();
   }
@@ -359,7 +361,7 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
   // first tile's weight stages before the programmatic-launch wait (constants)
   // (the row count is from the selection kernel, at least two launches back)
   int n_pre = 0;
-  if (warp == 4 && lane == 0 && static_cast<int>(blockIdx.x) < tiles) {
+  if (warp == WS_EPI_WARPS && lane == 0 && static_cast<int>(blockIdx.x) < tiles) {
     const int ft = blockIdx.x % n_ft, tt = blockIdx.x / n_ft;
     const int rows = min(BN_MAX, M - tt * BN_MAX);
     const int nbox = (((rows + 15) & ~15) + XBOX - 1) / XBOX;
@@ -372,7 +374,7 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
   pdl_wait();
   pdl_launch_dependents();
 
-  if (warp == 4) {
+  if (warp == WS_EPI_WARPS) {
     if (lane == 0) {
       const uint64_t pol_w = l2_policy_evict_first(), pol_x = l2_policy_evict_last();
       uint32_t stage = 0, phase = 0;
@@ -404,7 +406,7 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
         first = false;
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == WS_EPI_WARPS + 1) {
     if (lane == 0) {
       uint32_t stage = 0, phase = 0;
       int iter = 0;
@@ -442,8 +444,10 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
       }
     }
   } else {
-    // epilogue warps 0-3: TMEM lane 32 w + lane = tile-local output feature
-    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    // epilogue warps: TMEM lane 32 (w % 4) + lane = tile-local output feature; warp w
+    // takes the rows of half w / 4 of the tile (halves of a multiple of 16 rows)
+    const int quarter = warp & 3, half = warp >> 2;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     int iter = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++iter) {
       const int ft = tile % n_ft, tt = tile / n_ft;
@@ -455,15 +459,17 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
         break;
       }
       tc_fence_after();
-      const int f = ft * BM + warp * 32 + lane;
+      const int f = ft * BM + quarter * 32 + lane;
       const uint32_t acc = trow + static_cast<uint32_t>(b * BN_MAX);
-      for (int c0 = 0; c0 < rows; c0 += 16) {
+      const int hrows = ((rows + 31) / 32) * 16;
+      const int r_lo = half * hrows, r_hi = min(rows, r_lo + hrows);
+      for (int c0 = r_lo; c0 < r_hi; c0 += 16) {
         float v[16];
         tmem_ld16(acc + c0, v);
         if (f < a.n_out) {
 #pragma unroll
           for (int j = 0; j < 16; ++j)
-            if (c0 + j < rows) epilogue_store(a.epi, row0 + c0 + j, f, v[j]);
+            if (c0 + j < r_hi) epilogue_store(a.epi, row0 + c0 + j, f, v[j]);
         }
       }
       tc_fence_before();
@@ -473,7 +479,7 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == WS_EPI_WARPS + 1) {
     tc_fence_after();
     tmem_dealloc(tmem, 2 * BN_MAX);
   }

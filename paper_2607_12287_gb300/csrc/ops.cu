@@ -28,24 +28,44 @@ __device__ __forceinline__ bool is_cold(const ColdMask& m, int v) {
 
 // --------------------------------------------------------------------- patchify
 // patches[v*N + i][(ky*P + kx)*3 + c] = frame[v][py*P + ky][px*P + kx][c] - 128 (exact in
-// bf16).  One thread per (token, ky): P*3 contiguous bytes in, P*3 bf16 out.  Columns
-// P*P*3 .. kpad-1 stay zero (set once at allocation).
+// bf16).  When a patch row (P*3 bytes) has even length, one thread per pair of adjacent
+// columns: 2 bytes in, one bf16 pair out, so consecutive threads read and write
+// contiguous runs; otherwise one thread per (token, ky) row.  Columns P*P*3 .. kpad-1
+// stay zero (set once at allocation).
 __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __restrict__ patches,
                                 int sv, int img_h, int img_w, int P, int kpad) {
   pdl_wait();
   pdl_launch_dependents();
   const int gw = img_w / P, gh = img_h / P, N = gw * gh;
+  const int row = P * 3;
+  const long long stride = static_cast<long long>(gridDim.x) * blockDim.x;
+  if ((row & 1) == 0) {
+    const int pr = row / 2;  // column pairs per patch row
+    const long long total = static_cast<long long>(sv) * N * P * pr;
+    for (long long g = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; g < total; g += stride) {
+      const int j = static_cast<int>(g % pr);
+      const long long t2 = g / pr;
+      const int ky = static_cast<int>(t2 % P);
+      const long long tok = t2 / P;
+      const int v = static_cast<int>(tok / N), i = static_cast<int>(tok % N);
+      const int py = i / gw, px = i % gw;
+      const unsigned short b2 = *reinterpret_cast<const unsigned short*>(
+          frames + ((static_cast<size_t>(v) * img_h + py * P + ky) * img_w + px * P) * 3 + 2 * j);
+      *reinterpret_cast<__nv_bfloat162*>(patches + static_cast<size_t>(tok) * kpad + ky * row + 2 * j) =
+          __floats2bfloat162_rn(static_cast<float>(b2 & 0xFF) - 128.f, static_cast<float>(b2 >> 8) - 128.f);
+    }
+    return;
+  }
   const long long total = static_cast<long long>(sv) * N * P;
-  for (long long g = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; g < total;
-       g += static_cast<long long>(gridDim.x) * blockDim.x) {
+  for (long long g = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; g < total; g += stride) {
     const int ky = static_cast<int>(g % P);
     const long long tok = g / P;
     const int v = static_cast<int>(tok / N), i = static_cast<int>(tok % N);
     const int py = i / gw, px = i % gw;
     const uint8_t* src =
         frames + ((static_cast<size_t>(v) * img_h + py * P + ky) * img_w + px * P) * 3;
-    bf16* dst = patches + static_cast<size_t>(tok) * kpad + ky * P * 3;
-    for (int j = 0; j < P * 3; ++j) dst[j] = __float2bfloat16_rn(static_cast<float>(src[j]) - 128.f);
+    bf16* dst = patches + static_cast<size_t>(tok) * kpad + ky * row;
+    for (int j = 0; j < row; ++j) dst[j] = __float2bfloat16_rn(static_cast<float>(src[j]) - 128.f);
   }
 }
 
@@ -203,7 +223,8 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
 // -------------------------------------------------------------------- layernorm
 // One warp per row.  The row (up to 2048 floats) is read once into registers with
 // 128-bit loads; mean, centred second moment and the normalised output are computed
-// from registers in fp32.
+// from registers in fp32.  The affine parameters sit in shared memory (loaded before
+// the wait on the previous kernel), which leaves registers for more rows in flight.
 constexpr int LN_MAX_F4_PER_LANE = 16;
 
 // Optionally the input row is gathered (row src_rowtok[r] of x) and, with kAdd, a
@@ -220,15 +241,14 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, float* __restric
   const int n4 = dim / 4;
   // Before waiting on the previous kernel: the affine parameters (constant) and the row
   // count (written by the selection kernel, at least two launches back).
+  __shared__ float4 sg[LN_MAX_F4_PER_LANE * 32], sb[LN_MAX_F4_PER_LANE * 32];
   const float4* g4 = reinterpret_cast<const float4*>(gamma);
   const float4* b4 = reinterpret_cast<const float4*>(beta);
-  float4 g[LN_MAX_F4_PER_LANE], bb[LN_MAX_F4_PER_LANE];
-#pragma unroll
-  for (int i = 0; i < LN_MAX_F4_PER_LANE; ++i) {
-    const int c = lane + 32 * i;
-    g[i] = c < n4 ? g4[c] : make_float4(0.f, 0.f, 0.f, 0.f);
-    bb[i] = c < n4 ? b4[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int c = threadIdx.x; c < n4; c += blockDim.x) {
+    sg[c] = g4[c];
+    sb[c] = b4[c];
   }
+  __syncthreads();
   const int rows = *nrows;
   pdl_wait();
   pdl_launch_dependents();
@@ -264,11 +284,9 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, float* __restric
     for (int i = 0; i < LN_MAX_F4_PER_LANE; ++i) {
       const int c = lane + 32 * i;
       if (c < n4) {
-        const float4 u = v[i];
-        yr[2 * c] = __floats2bfloat162_rn(g[i].x * (u.x - mean) * rstd + bb[i].x,
-                                          g[i].y * (u.y - mean) * rstd + bb[i].y);
-        yr[2 * c + 1] = __floats2bfloat162_rn(g[i].z * (u.z - mean) * rstd + bb[i].z,
-                                              g[i].w * (u.w - mean) * rstd + bb[i].w);
+        const float4 u = v[i], g = sg[c], bb = sb[c];
+        yr[2 * c] = __floats2bfloat162_rn(g.x * (u.x - mean) * rstd + bb.x, g.y * (u.y - mean) * rstd + bb.y);
+        yr[2 * c + 1] = __floats2bfloat162_rn(g.z * (u.z - mean) * rstd + bb.z, g.w * (u.w - mean) * rstd + bb.w);
       }
     }
   }
@@ -496,9 +514,10 @@ __global__ void __launch_bounds__(ATT_WARPS * 32)
 
 cudaError_t launch_patchify(const uint8_t* frames, bf16* patches, int sv, int img_h, int img_w,
                             int patch, int kpad, cudaStream_t s) {
-  const long long total = static_cast<long long>(sv) * (img_h / patch) * (img_w / patch) * patch;
+  long long total = static_cast<long long>(sv) * (img_h / patch) * (img_w / patch) * patch;
+  if ((patch * 3) % 2 == 0) total *= patch * 3 / 2;
   const long long blocks = (total + 255) / 256;
-  const int grid = static_cast<int>(blocks < 4096 ? blocks : 4096);
+  const int grid = static_cast<int>(blocks < 8192 ? blocks : 8192);
   return launch_ex(patchify_kernel, dim3(grid), dim3(256), 0, s, 1, frames, patches, sv, img_h, img_w, patch, kpad);
 }
 
