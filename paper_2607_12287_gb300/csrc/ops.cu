@@ -39,15 +39,16 @@ __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __rest
   const int gw = img_w / P, gh = img_h / P, N = gw * gh;
   const int row = P * 3;
   const long long stride = static_cast<long long>(gridDim.x) * blockDim.x;
-  if ((row & 1) == 0) {
+  if ((row & 1) == 0 && static_cast<long long>(sv) * N * P * (row / 2) < (1LL << 30)) {
+    // 32-bit index arithmetic (the divisions dominate this kernel's instruction count)
     const int pr = row / 2;  // column pairs per patch row
-    const long long total = static_cast<long long>(sv) * N * P * pr;
-    for (long long g = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; g < total; g += stride) {
-      const int j = static_cast<int>(g % pr);
-      const long long t2 = g / pr;
-      const int ky = static_cast<int>(t2 % P);
-      const long long tok = t2 / P;
-      const int v = static_cast<int>(tok / N), i = static_cast<int>(tok % N);
+    const int total = sv * N * P * pr;
+    for (int g = blockIdx.x * blockDim.x + threadIdx.x; g < total; g += static_cast<int>(stride)) {
+      const int j = g % pr;
+      const int t2 = g / pr;
+      const int ky = t2 % P;
+      const int tok = t2 / P;
+      const int v = tok / N, i = tok % N;
       const int py = i / gw, px = i % gw;
       const unsigned short b2 = *reinterpret_cast<const unsigned short*>(
           frames + ((static_cast<size_t>(v) * img_h + py * P + ky) * img_w + px * P) * 3 + 2 * j);
