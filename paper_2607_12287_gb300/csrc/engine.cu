@@ -133,8 +133,12 @@ struct ivit_handle {
   std::vector<uint8_t> cold;
   int64_t launches = 0;
 
-  // Persistent encoder (all blocks in one cooperative launch) for small row tiles.
+  // Persistent encoder (all blocks in one cooperative launch) for small encoders: it runs
+  // the full encodes; incremental calls run it only when forced (persistent_inc), since
+  // the kernel chain is faster for a few updated rows (its tensor-core attention against
+  // the persistent kernel's SIMT attention phase).
   bool persistent = false;
+  bool persistent_inc = false;
   size_t pt_smem = 0;
   int pt_grid = 0;
   void* pt_mem = nullptr;  // device: tensor maps, layer parameters, partials, barrier words
@@ -237,12 +241,14 @@ GemmPlan plan_gemm(int num_sms, int bn, int n_out, int k, int m_expected) {
 // Prepares the persistent encoder when its shared memory fits (attention keeps a whole
 // view's keys and values of one head resident, so N * head_dim is bounded).
 int setup_persistent(ivit_handle* h) {
-  // IVIT_PATH=kernels / IVIT_PATH=persistent override the choice made from the shape.
-  // Default: small encoders (dim <= 384), whose per-layer kernels are launch-bound.
+  // IVIT_PATH=kernels / IVIT_PATH=persistent (every call) override the choice made from
+  // the shape.  Default: the full encodes of small encoders (dim <= 384), whose
+  // per-layer kernels are launch-bound at every row of every view.
   const char* path = std::getenv("IVIT_PATH");
   if (path && std::strcmp(path, "kernels") == 0) return IVIT_OK;
   if (h->cfg.mlp_tokens == IVIT_MLP_ALL) return IVIT_OK;  // the kernel chain runs that reading
-  if (!(path && std::strcmp(path, "persistent") == 0) && h->D > 384) return IVIT_OK;
+  const bool forced = path && std::strcmp(path, "persistent") == 0;
+  if (!forced && h->D > 384) return IVIT_OK;
   const int dh = h->D / h->H;
   const size_t smem = ivit::persistent_smem_bytes(h->N, dh);
   if (smem > 227 * 1024 || h->D > 2048 || h->N > 256) return IVIT_OK;
@@ -323,6 +329,7 @@ int setup_persistent(ivit_handle* h) {
   h->pt_smem = smem;
   h->pt_grid = grid;
   h->persistent = true;
+  h->persistent_inc = forced;
   return IVIT_OK;
 }
 
@@ -804,7 +811,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
                                  c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
   ++h->launches;
 
-  if (h->persistent) {
+  if (h->persistent && (full || h->persistent_inc)) {
     IVIT_CK(h, cudaMemsetAsync(h->pt_args.gbar, 0, 4 * sizeof(unsigned), s));
     IVIT_CK(h, ivit::launch_persistent(h->pt_args, h->pt_grid, h->pt_smem, s));
     ++h->launches;

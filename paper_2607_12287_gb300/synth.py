@@ -296,7 +296,9 @@ def stream_rects(shape: EncoderShape, views: Sequence[ViewScene], n_frames: int,
 def stream_moving_square(shape: EncoderShape, n_frames: int, seed: int,
                          size: int = 48, y0: int = 88, x0: int = 8,
                          step: int = 16) -> Iterator[np.ndarray]:
-    """Uniform-noise background fixed; a solid square moves ``step`` px/frame in x.
+    """Uniform-noise background fixed; a solid square moves ``step`` px/frame in x and
+    turns back at the image's right edge (and again at ``x0``), so every frame of an
+    arbitrarily long stream has motion.
 
     The square's colour has every channel in [0, 63] or [192, 255] (far from the
     background mean).  Every pixel outside the square gets fresh +-1 noise per frame.
@@ -307,9 +309,12 @@ def stream_moving_square(shape: EncoderShape, n_frames: int, seed: int,
     bg = rng.integers(0, 256, size=(H, W, 3), dtype=np.uint8)
     lo = rng.integers(0, 64, size=3)
     colour = np.where(rng.random(3) < 0.5, lo, 192 + lo).astype(np.uint8)
+    n_pos = max(1, (W - size - x0) // step + 1)  # left edges with the whole square inside
+    period = max(1, 2 * (n_pos - 1))
     for t in range(n_frames):
         img = _pm1_noise(rng, bg)
-        x = x0 + step * t
+        k = t % period
+        x = x0 + step * (k if k < n_pos else period - k)
         img[y0:y0 + size, max(x, 0):min(x + size, W)] = colour
         yield img[None]
 
