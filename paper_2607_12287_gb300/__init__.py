@@ -98,6 +98,30 @@ def _ptr(t) -> Optional[int]:
     return t.data_ptr()
 
 
+def _require(t, name: str, dtype_name: str, numel: int) -> None:
+    """Rejects a tensor that the kernels would misread or index out of bounds: one in host
+    memory, of another dtype (``dtype_name`` is the torch dtype's name, e.g. "uint8"), a
+    non-contiguous view, or one with fewer than ``numel`` elements.  ``None`` (an optional
+    output) and raw integer pointers pass unchecked: the caller vouches for those."""
+    if t is None or isinstance(t, int):
+        return
+    if isinstance(t, np.ndarray):
+        raise TypeError(f"{name}: a numpy array (host memory); a CUDA tensor is required")
+    if t.device.type != "cuda":
+        raise ValueError(f"{name}: tensor on {t.device}; a CUDA tensor is required")
+    if str(t.dtype) != "torch." + dtype_name:
+        raise TypeError(f"{name}: dtype {t.dtype}, expected torch.{dtype_name}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name}: not contiguous")
+    if t.numel() < numel:
+        raise ValueError(f"{name}: {t.numel()} elements, the call needs {numel}")
+
+
+# handle -> (views, frame bytes per view, tokens per view, width), registered at create so
+# that the entry points can check the tensors they are given against the encoder's sizes
+_dims = {}
+
+
 def _stream(stream) -> Optional[int]:
     if stream is None:
         import torch
@@ -136,15 +160,28 @@ def ivit_create(cfg: IvitConfig, weights_u16: np.ndarray) -> int:
     w = np.ascontiguousarray(weights_u16, dtype=np.uint16)
     h = C.c_void_p()
     _check(load().ivit_create(C.byref(cfg), w.ctypes.data, C.byref(h)), None)
+    n_tok = (cfg.img_h // cfg.patch) * (cfg.img_w // cfg.patch)
+    _dims[h.value] = (cfg.n_streams * cfg.n_views, cfg.img_h * cfg.img_w * 3, n_tok, cfg.dim)
     return h.value
 
 
+def _check_call(h: int, frames, tokens_out, changed_count=None) -> None:
+    if h not in _dims:
+        return  # a handle created outside this module: sizes unknown here
+    sv, fbytes, n_tok, dim = _dims[h]
+    _require(frames, "frames", "uint8", sv * fbytes)
+    _require(tokens_out, "tokens_out", "bfloat16", sv * n_tok * dim)
+    _require(changed_count, "changed_count", "int32", sv)
+
+
 def ivit_encode_full(h: int, frames, tokens_out=None, stream=None) -> None:
+    _check_call(h, frames, tokens_out)
     _check(load().ivit_encode_full(h, _ptr(frames), _ptr(tokens_out), _stream(stream)), h)
 
 
 def ivit_encode_incremental(h: int, frames, tokens_out=None, changed_count=None,
                             stream=None) -> None:
+    _check_call(h, frames, tokens_out, changed_count)
     _check(load().ivit_encode_incremental(h, _ptr(frames), _ptr(tokens_out),
                                           _ptr(changed_count), _stream(stream)), h)
 
@@ -180,6 +217,7 @@ def ivit_last_launch_count(h: int) -> int:
 
 
 def ivit_destroy(h: int) -> None:
+    _dims.pop(h, None)
     load().ivit_destroy(h)
 
 
@@ -187,6 +225,12 @@ def ivit_select_noalloc(e_cur, e_ref, n_views: int, n_tok: int, dim: int, select
                         threshold: float, topk: int, idx_out, counts_out, stream=None) -> None:
     """Selection without device allocation (scratch in a fixed device array); for callers
     that cannot allocate, e.g. while a stream is being captured into a CUDA graph."""
+    if 0 < n_views * n_tok <= IVIT_NOALLOC_MAX_TOKENS and dim > 0:
+        # (other sizes are rejected by the library before any device work)
+        _require(e_cur, "e_cur", "float32", n_views * n_tok * dim)
+        _require(e_ref, "e_ref", "float32", n_views * n_tok * dim)
+        _require(idx_out, "idx_out", "int32", n_views * n_tok)
+        _require(counts_out, "counts_out", "int32", n_views)
     _check(load().ivit_select_noalloc(_ptr(e_cur), _ptr(e_ref), n_views, n_tok, dim, select_mode,
                                       threshold, topk, _ptr(idx_out), _ptr(counts_out),
                                       _stream(stream)), None)
@@ -195,7 +239,13 @@ def ivit_select_noalloc(e_cur, e_ref, n_views: int, n_tok: int, dim: int, select
 def ivit_action_combine(x0, v0, v7, alpha, beta, b, xT, stream=None) -> None:
     """Eq. 9 action combine on device tensors: x0, v0, v7, b (or None), xT fp32 [B, A];
     alpha, beta fp32 [B]."""
-    B, A = (int(x0.shape[0]), int(x0.shape[1])) if x0.dim() == 2 else (0, 0)
+    if x0.dim() != 2:
+        raise ValueError(f"x0: shape {tuple(x0.shape)}, expected [batch, action width]")
+    B, A = int(x0.shape[0]), int(x0.shape[1])
+    for t, name in ((x0, "x0"), (v0, "v0"), (v7, "v7"), (b, "b"), (xT, "xT")):
+        _require(t, name, "float32", B * A)
+    _require(alpha, "alpha", "float32", B)
+    _require(beta, "beta", "float32", B)
     _check(load().ivit_action_combine(_ptr(x0), _ptr(v0), _ptr(v7), _ptr(alpha), _ptr(beta),
                                       _ptr(b) if b is not None else None, B, A, _ptr(xT),
                                       _stream(stream)), None)

@@ -197,7 +197,8 @@ def _smooth_texture(rng: np.random.Generator, h: int, w: int, cell: int = 16,
     smooth = (c00 * (1 - fy) * (1 - fx) + c01 * (1 - fy) * fx
               + c10 * fy * (1 - fx) + c11 * fy * fx)
     img = 128.0 + smooth + rng.uniform(-grain, grain, size=(h, w, 3))
-    return np.clip(np.rint(img), 0, 255).astype(np.uint8)
+    # (fancy indexing above leaves the axes in another memory order: frames are row-major)
+    return np.ascontiguousarray(np.clip(np.rint(img), 0, 255).astype(np.uint8))
 
 
 def _pm1_noise(rng: np.random.Generator, img: np.ndarray) -> np.ndarray:
