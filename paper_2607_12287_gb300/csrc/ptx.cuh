@@ -309,6 +309,11 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 }
 
 // ------------------------------------------------------ programmatic dependent launch
+// Every tcgen05 kernel allocates its TMEM columns before pdl_wait and calls
+// pdl_launch_dependents only after it.  So at most two grids overlap on an SM, every CTA
+// of the earlier grid already holds its columns when the later grid's CTAs allocate, and
+// an allocation can only wait for a CTA that is not waiting for it (no TMEM deadlock
+// between a kernel and the one launched early behind it).
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
