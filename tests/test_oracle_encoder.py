@@ -16,6 +16,10 @@ from tests import restate
 SHAPES = [
     synth.EncoderShape(32, 48, 8, 32, 2, 2, 64, synth.GELU_TANH),
     synth.EncoderShape(28, 28, 7, 48, 3, 3, 80, synth.GELU_ERF),
+    # degenerate shapes: one token per view (attention over a single key returns its
+    # value), and one-pixel patches (K = 3) with single-pixel-wide heads of 6
+    synth.EncoderShape(8, 8, 8, 16, 2, 1, 32, synth.GELU_TANH),
+    synth.EncoderShape(4, 6, 1, 24, 2, 4, 40, synth.GELU_ERF),
 ]
 
 
@@ -48,6 +52,7 @@ def test_incremental_vs_masked_restatement(oracle_mod, shape):
     orc = oracle_mod.Oracle(shape, w, 2, 1)
     orc.encode_full(frames[0])
     state = []
+    updated = 0
     for v in range(2):
         t64, K64, V64, e64 = restate.full(shape, W, frames[0][v])
         state.append([t64, K64, V64, e64])
@@ -66,7 +71,8 @@ def test_incremental_vs_masked_restatement(oracle_mod, shape):
             assert rel(tok[v], t64) < 1e-5
             for l in range(shape.depth):
                 assert rel(orc.cache("K", l)[v], K64[l]) < 1e-5
-        assert counts.sum() > 0
+        updated += int(counts.sum())
+    assert updated > 0  # the stream exercised the incremental path
 
 
 def test_all_changed_incremental_equals_full_bitwise(oracle_mod):
