@@ -152,14 +152,19 @@ int ivit_profile_read(ivit_handle* h, double* gemm_ms_total, int64_t* gemm_launc
 int ivit_device_status(ivit_handle* h, void* stream);
 
 /* Execution paths (chosen at create; the environment variable IVIT_PATH=kernels or
- * IVIT_PATH=persistent overrides the default): one kernel per operation, chained with
- * programmatic dependent launch and replayed as a CUDA graph (default for dim > 384),
- * or every transformer block of a call in one persistent cooperative kernel with grid
- * barriers (default for dim <= 384, where per-operation launches dominate). */
+ * IVIT_PATH=persistent selects one for every call): one kernel per operation, chained
+ * with programmatic dependent launch and replayed as a CUDA graph (every incremental
+ * call, and the full encodes for dim > 384), or every transformer block of a call in
+ * one persistent cooperative kernel with grid barriers (the full encodes for
+ * dim <= 384, where per-operation launches dominate).  Both give the same result. */
 
 /* Number of the library's kernel launches made by the last encode call. */
 int64_t ivit_last_launch_count(const ivit_handle* h);
 
+/* Releases the handle and every device buffer, CUDA graph and stream it owns (weights,
+ * caches, workspaces).  The device memory is freed with cudaFree, which waits for work
+ * in flight on the device; the caller must not use `h` from another thread meanwhile or
+ * afterwards.  NULL does nothing. */
 void ivit_destroy(ivit_handle* h);
 
 /* Token selection that allocates nothing.  The paper has no counterpart: this entry
