@@ -27,6 +27,26 @@ def declared_entry_points():
     return sorted(set(re.findall(r"\b(ivit_[a-z_]+)\s*\(", text)))
 
 
+def test_every_entry_point_is_documented_in_the_header():
+    # each declaration (or group of adjacent declarations) follows a comment block that
+    # states the operation, argument layouts, ownership and errors
+    lines = open(os.path.join(ROOT, "include", "ivit.h")).read().splitlines()
+    decl = re.compile(r"^[A-Za-z].*\b(ivit_[a-z_]+)\s*\(")
+    undocumented = []
+    for i, line in enumerate(lines):
+        m = decl.match(line)
+        if not m:
+            continue
+        j = i - 1
+        # skip earlier declarations of the group (and their continuation lines) and macros
+        while j >= 0 and (lines[j].startswith("#define") or lines[j].startswith(" ") and not
+                          lines[j].strip().endswith("*/") or decl.match(lines[j])):
+            j -= 1
+        if j < 0 or not lines[j].rstrip().endswith("*/"):
+            undocumented.append(m.group(1))
+    assert not undocumented, f"entry points without a comment block: {undocumented}"
+
+
 def test_header_declares_the_binding_names(pkg):
     assert declared_entry_points() == sorted(pkg.EXPORTED)
 
