@@ -125,7 +125,7 @@ int ivit_encode_incremental(ivit_handle* h, const uint8_t* frames_dev,
 
 /* Copies the ascending updated-token list of view `sv` from the last encode call:
  * idx_dev int32 [N] (first *count entries valid), count_dev int32 [1] (either may be
- * NULL).  Enqueued on `stream`. */
+ * NULL).  Enqueued on `stream`.  IVIT_ERR_ARG if sv is outside [0, SV). */
 int ivit_get_changed(ivit_handle* h, int sv, int32_t* idx_dev, int32_t* count_dev,
                      void* stream);
 
@@ -133,11 +133,13 @@ int ivit_get_changed(ivit_handle* h, int sv, int32_t* idx_dev, int32_t* count_de
  * of `layer`, 2 final-token cache (all bf16 [SV][N][D]), 3 reference score vectors
  * (patch embeddings or first-layer keys, fp32 [SV][N][D]), 4 attention-block outputs of
  * `layer` (fp32 [SV][N][D], mlp_tokens = IVIT_MLP_ALL only).  dst_dev must hold that
- * many bytes. */
+ * many bytes.  IVIT_ERR_ARG for a NULL destination, an unknown `which` (4 without that
+ * reading) or, for 0, 1 and 4, a layer outside [0, L). */
 int ivit_get_cache(ivit_handle* h, int which, int layer, void* dst_dev, void* stream);
 
 /* Marks the views of camera stream `stream_index` (all streams if -1) cold: the next
- * incremental call recomputes every token of those views.  Host-side only. */
+ * incremental call recomputes every token of those views.  Host-side only.
+ * IVIT_ERR_ARG if stream_index is outside [-1, n_streams). */
 int ivit_reset(ivit_handle* h, int stream_index);
 
 /* Kernel timing hook: when enabled, every launch of the dominant kernel family (the
