@@ -1,0 +1,66 @@
+"""Host-side pieces of bench.py that need no GPU: the DRAM-traffic ratio taken from the
+committed ncu summary (and dropped once the profiled kernel source changes), and the
+clock/throttle summary parsed from nvidia-smi samples."""
+import hashlib
+import os
+
+import bench
+
+GEMM_SRC = os.path.join(bench.ROOT, "paper_2607_12287_gb300", "csrc", "gemm.cu")
+
+
+def _tree(tmp_path, src: str, ratio: float, digest: str):
+    (tmp_path / "profiles").mkdir()
+    (tmp_path / "profiles" / "gemm_tc_kernel_so400m_224_1view.md").write_text(
+        f"traffic_to_algorithmic_ratio: {ratio}\ngemm_tc_kernel_source_sha256: {digest}\n")
+    csrc = tmp_path / "paper_2607_12287_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    (csrc / "gemm.cu").write_text(src)
+
+
+def test_traffic_ratio_follows_the_profiled_source(tmp_path, monkeypatch):
+    src = open(GEMM_SRC).read()
+    cut = src.find("// Many-tile form")
+    assert cut > 0
+    digest = hashlib.sha256(src[:cut].encode()).hexdigest()
+    _tree(tmp_path, src, 0.99, digest)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.gemm_traffic_ratio() == 0.99
+    # a change below the profiled kernel (the warp-specialised form) keeps the ratio
+    (tmp_path / "paper_2607_12287_gb300" / "csrc" / "gemm.cu").write_text(src + "\n// tail\n")
+    assert bench.gemm_traffic_ratio() == 0.99
+    # a change inside the profiled kernel drops it
+    (tmp_path / "paper_2607_12287_gb300" / "csrc" / "gemm.cu").write_text("// edit\n" + src)
+    assert bench.gemm_traffic_ratio() is None
+
+
+def test_traffic_ratio_absent_summary(tmp_path, monkeypatch):
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.gemm_traffic_ratio() is None
+
+
+def test_clock_summary_parses_samples_and_reasons(tmp_path):
+    csv = tmp_path / "clocks.csv"
+    csv.write_text(
+        "0, 2070, 2070, 900.1, 0x0, Not Active, Not Active, Not Active, Not Active\n"
+        "0, 2055, 2070, 1390.5, 0x4, Not Active, Not Active, Not Active, Active\n"
+        "0, 2070, 2070, 1201.0, 0x0, Not Active, Not Active, Not Active, Not Active\n"
+        "garbage line\n")
+    s = bench.ClockSampler(0)
+    s.proc, s.path = object(), str(csv)  # as if nvidia-smi had written the file
+    out = s.summary()
+    assert out == {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "samples": 3, "reasons": ["sw_power_cap"]}
+    assert not csv.exists()  # the sample file is removed once read
+
+
+def test_clock_summary_without_nvidia_smi():
+    s = bench.ClockSampler(0)
+    assert s.summary() is None
+
+
+def test_describe_names_the_workload():
+    from paper_2607_12287_gb300 import synth
+    d = bench.describe(synth.WORKLOADS["so400m_224_1view"])
+    assert d["workload"] == "so400m_224_1view" and d["views"] == 1
+    assert "dim 1152" in d["encoder"] and "27 layers" in d["encoder"]
+    assert bench.describe(synth.sweep_workload(0.25))["selection"] == "top-64"
