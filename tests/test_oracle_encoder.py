@@ -187,3 +187,33 @@ def test_selection_equals_repainted_patches(oracle_mod):
         truth = synth.pixel_changed_patches(prev, cur, shape.patch)
         for v in range(2):
             np.testing.assert_array_equal(idx[v, :counts[v]], np.nonzero(truth[v])[0])
+
+
+def test_so400m_layer_shape_on_the_bench_stream(oracle_mod):
+    # the SigLIP-So400m block (D 1152, 16 heads of 72, MLP 4304, 256 tokens of 14-px
+    # patches) with two of its 27 layers, on the bench's camera stream: full encode and
+    # two incremental frames against the fp64 restatement
+    import dataclasses
+    shape = dataclasses.replace(synth.SO400M_224, depth=2)
+    w = synth.make_weights(shape, 0)
+    W = restate.weights64(shape, w)
+    frames = list(synth.WORKLOADS["so400m_224_1view"].frames(3))
+    orc = oracle_mod.Oracle(shape, w, 1, 1)
+    tok = orc.encode_full(frames[0])
+    t64, K64, V64, e = restate.full(shape, W, frames[0][0])
+    assert rel(tok[0], t64) < 1e-5
+    for f in frames[1:]:
+        tok, counts, idx, sims = orc.encode_incremental(f)
+        e1 = restate.embed(shape, W, f[0])
+        s64 = torch.nn.functional.cosine_similarity(e1, e, dim=1).numpy()
+        np.testing.assert_allclose(sims[0], s64, atol=1e-5)
+        mask = s64 < 0.98
+        assert np.abs(s64 - 0.98).min() > 1e-3
+        np.testing.assert_array_equal(idx[0, :counts[0]], np.nonzero(mask)[0])
+        assert 0 < counts[0] < shape.n_tokens
+        K64, V64, t64 = restate.run_rows(shape, W, e1, mask, K64, V64, t64)
+        e = e1
+        assert rel(tok[0], t64) < 1e-5
+        for l in range(shape.depth):
+            assert rel(orc.cache("K", l)[0], K64[l]) < 1e-5
+            assert rel(orc.cache("V", l)[0], V64[l]) < 1e-5
