@@ -217,3 +217,28 @@ def test_so400m_layer_shape_on_the_bench_stream(oracle_mod):
         for l in range(shape.depth):
             assert rel(orc.cache("K", l)[0], K64[l]) < 1e-5
             assert rel(orc.cache("V", l)[0], V64[l]) < 1e-5
+
+
+def test_so400m_448_layer_shape_on_the_batched_stream(oracle_mod):
+    # 448 px frames (1024 tokens: attention over 1024 keys) with one So400m layer, on
+    # view 0 of the batched 16 x 2 stream: full encode and one incremental frame
+    import dataclasses
+    wl = synth.WORKLOADS["so400m_448_16x2"]
+    shape = dataclasses.replace(wl.shape, depth=1)
+    w = synth.make_weights(shape, 0)
+    W = restate.weights64(shape, w)
+    f0, f1 = (f[:1] for f in wl.frames(2))
+    orc = oracle_mod.Oracle(shape, w, 1, 1)
+    tok = orc.encode_full(f0)
+    t64, K64, V64, e = restate.full(shape, W, f0[0])
+    assert rel(tok[0], t64) < 1e-5
+    tok, counts, idx, sims = orc.encode_incremental(f1)
+    e1 = restate.embed(shape, W, f1[0])
+    s64 = torch.nn.functional.cosine_similarity(e1, e, dim=1).numpy()
+    mask = s64 < 0.98
+    assert np.abs(s64 - 0.98).min() > 1e-3
+    np.testing.assert_array_equal(idx[0, :counts[0]], np.nonzero(mask)[0])
+    assert 0 < counts[0] < shape.n_tokens
+    K64, V64, t64 = restate.run_rows(shape, W, e1, mask, K64, V64, t64)
+    assert rel(tok[0], t64) < 1e-5
+    assert rel(orc.cache("K", 0)[0], K64[0]) < 1e-5
