@@ -242,3 +242,28 @@ def test_so400m_448_layer_shape_on_the_batched_stream(oracle_mod):
     K64, V64, t64 = restate.run_rows(shape, W, e1, mask, K64, V64, t64)
     assert rel(tok[0], t64) < 1e-5
     assert rel(orc.cache("K", 0)[0], K64[0]) < 1e-5
+
+
+def test_vit_tiny_on_the_square_stream(oracle_mod):
+    # the whole ViT-Tiny encoder (12 layers, 3 heads of 64, erf GELU, 196 tokens) on the
+    # moving-square stream: full encode, then incremental frames against the restatement
+    wl = synth.WORKLOADS["vit_tiny_224_square"]
+    shape = wl.shape
+    w = synth.make_weights(shape, 0)
+    W = restate.weights64(shape, w)
+    frames = list(wl.frames(4))
+    orc = oracle_mod.Oracle(shape, w, 1, 1)
+    tok = orc.encode_full(frames[0])
+    t64, K64, V64, e = restate.full(shape, W, frames[0][0])
+    assert rel(tok[0], t64) < 1e-5
+    for prev, f in zip(frames, frames[1:]):
+        tok, counts, idx, sims = orc.encode_incremental(f)
+        e1 = restate.embed(shape, W, f[0])
+        mask = torch.nn.functional.cosine_similarity(e1, e, dim=1).numpy() < 0.98
+        truth = synth.pixel_changed_patches(prev, f, shape.patch)[0]
+        np.testing.assert_array_equal(mask, truth)
+        np.testing.assert_array_equal(idx[0, :counts[0]], np.nonzero(mask)[0])
+        K64, V64, t64 = restate.run_rows(shape, W, e1, mask, K64, V64, t64)
+        e = e1
+        assert rel(tok[0], t64) < 1e-5
+        assert rel(orc.cache("V", shape.depth - 1)[0], V64[-1]) < 1e-5
