@@ -48,3 +48,29 @@ def test_moving_square_path():
     assert lefts[11:21] == [8 + 16 * (20 - t) for t in range(11, 21)]
     assert all(w == 48 for _, w in spans)
     assert max(lefts) + 48 <= wl.shape.img_w
+
+
+def _fractions(wl, n_frames):
+    frames = list(wl.frames(n_frames))
+    counts = np.array([synth.pixel_changed_patches(a, b, wl.shape.patch).sum(1)
+                       for a, b in zip(frames, frames[1:])])  # [steps, views]
+    return counts / wl.shape.n_tokens
+
+
+def test_bench_stream_is_ten_percent_dynamic():
+    f = _fractions(synth.WORKLOADS["so400m_224_1view"], 64)
+    assert 0.09 <= f.mean() <= 0.11
+    assert f.min() > 0 and f.max() <= 0.15
+
+
+def test_three_view_stream_targets_5_15_30_percent():
+    f = _fractions(synth.WORKLOADS["so400m_224_3view"], 64).mean(0)
+    assert 0.04 <= f[0] <= 0.08 and 0.14 <= f[1] <= 0.20 and 0.23 <= f[2] <= 0.31, f
+
+
+def test_batched_448_stream_mix():
+    f = _fractions(synth.WORKLOADS["so400m_448_16x2"], 12)
+    assert f.shape[1] == 32
+    assert 0.06 <= f.mean() <= 0.14
+    assert f.min() >= 0.01 and f.max() <= 0.25
+    assert f.mean(0).std() > 0.02  # views differ (per-stream random walks of object counts)
