@@ -94,3 +94,45 @@ def test_null_handle_calls_return_arg_error(pkg):
     assert L.ivit_get_changed(None, 0, None, None, None) == pkg.IVIT_ERR_ARG
     assert L.ivit_device_status(None, None) == pkg.IVIT_ERR_ARG
     L.ivit_destroy(None)
+
+
+C_CLIENT = r"""
+#include <stdio.h>
+#include <string.h>
+#include "ivit.h"
+
+int main(void) {
+  ivit_config c;
+  memset(&c, 0, sizeof c);
+  c.img_h = 224; c.img_w = 224; c.patch = 14; c.dim = 1152; c.depth = 27; c.heads = 16;
+  c.mlp_dim = 4304; c.n_streams = 1; c.n_views = 1; c.ln_eps = 1e-6f;
+  c.gelu = IVIT_GELU_TANH; c.select_mode = IVIT_SEL_THRESHOLD; c.threshold = 0.98f;
+  c.ref_mode = IVIT_REF_PREV_FRAME; c.score_source = IVIT_SCORE_EMBED;
+  c.schedule = IVIT_SCHED_INCREMENTAL; c.mlp_tokens = IVIT_MLP_UPDATED;
+  printf("%zu\n", ivit_weights_size(&c));
+  c.dim = 100; /* not a multiple of 64 */
+  ivit_handle* h = (ivit_handle*)0;
+  int r = ivit_create(&c, (const uint16_t*)0, &h);
+  printf("%d %d %s\n", r, h == (ivit_handle*)0, ivit_last_error((const ivit_handle*)0));
+  printf("%d\n", ivit_reset((ivit_handle*)0, 0));
+  ivit_destroy((ivit_handle*)0);
+  return 0;
+}
+"""
+
+
+def test_header_is_plain_c_and_links(pkg, tmp_path):
+    # a C99 client compiled against include/ivit.h and linked with the library; it calls
+    # only entry points that need no device
+    src = tmp_path / "client.c"
+    src.write_text(C_CLIENT)
+    exe = tmp_path / "client"
+    lib_dir = os.path.dirname(pkg.LIB_PATH)
+    subprocess.run(["gcc", "-std=c99", "-Wall", "-Wextra", "-Werror", "-I", os.path.join(ROOT, "include"),
+                    str(src), "-o", str(exe), "-L", lib_dir, "-l:libivit.so", f"-Wl,-rpath,{lib_dir}"],
+                   check=True, capture_output=True, text=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.splitlines()
+    assert int(out[0]) == synth.weight_count(synth.SO400M_224)
+    code, null_out, msg = out[1].split(" ", 2)
+    assert int(code) == pkg.IVIT_ERR_SHAPE and null_out == "1" and "64" in msg
+    assert int(out[2]) == pkg.IVIT_ERR_ARG
