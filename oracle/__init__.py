@@ -2,7 +2,8 @@
 
 TEST INFRASTRUCTURE ONLY: the oracle is a plain, slow CPU restatement of temporal
 token reuse (Sec. III-B) that the CUDA library is checked against.  Only ``tests/``,
-``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline leg may import it.
+``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline leg and reference arm (both
+time it on the host cores) may import it.
 """
 from __future__ import annotations
 

@@ -3,8 +3,8 @@
  *
  * TEST INFRASTRUCTURE ONLY.  This is a plain, slow CPU restatement of the method,
  * used to check the CUDA library.  Only the test suite, the smoke check and the
- * bench's CPU-baseline leg load it; the library never calls it and shares no code,
- * header or constant with it.
+ * bench's CPU-baseline leg and reference arm (both time it on the host cores) load
+ * it; the library never calls it and shares no code, header or constant with it.
  *
  * Storage is fp32; every dot product, layer-norm statistic and softmax sum is
  * accumulated in double.  The change score (Eq. 3) is computed in fp32, the
