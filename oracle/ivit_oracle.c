@@ -156,15 +156,6 @@ float orc_gelu(float x, int mode) {
   return (float)(0.5 * xd * (1.0 + tanh(c * (xd + 0.044715 * xd * xd * xd))));
 }
 
-static float round_bf16(float x) {
-  uint32_t u;
-  memcpy(&u, &x, sizeof u);
-  u = (u + 0x7FFFu + ((u >> 16) & 1u)) & 0xFFFF0000u; /* nearest, ties to even */
-  float y;
-  memcpy(&y, &u, sizeof y);
-  return y;
-}
-
 void orc_layer0_keys(const float* e, const float* pos, const float* ln_g, const float* ln_b,
                      const float* W_K, const float* b_K, int n, int D, float eps, float* k) {
 #pragma omp parallel for schedule(static)
@@ -173,7 +164,6 @@ void orc_layer0_keys(const float* e, const float* pos, const float* ln_g, const 
     float* xn = (float*)malloc(sizeof(float) * (size_t)D);
     for (int d = 0; d < D; ++d) x[d] = e[(size_t)i * D + d] + pos[(size_t)i * D + d];
     orc_layernorm(x, ln_g, ln_b, D, eps, xn);
-    for (int d = 0; d < D; ++d) xn[d] = round_bf16(xn[d]);
     orc_linear(xn, W_K, b_K, D, D, k + (size_t)i * D);
     free(x);
     free(xn);

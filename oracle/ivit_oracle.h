@@ -91,9 +91,9 @@ void orc_layernorm(const float* x, const float* g, const float* b, int n, float 
 void orc_linear(const float* x, const float* W, const float* b, int n_in, int n_out,
                 float* y);
 float orc_gelu(float x, int mode);
-/* Eq. 3 key vectors of the first layer for n tokens: k[i] = W_K bf16(LN1(e[i] + pos[i]))
- * + b_K, with the LN output rounded to bf16 (the precision the GPU path computes the
- * keys in, so both sides take the selection decision alike).  W_K [D][D]. */
+/* Eq. 3 key vectors of the first layer for n tokens: k[i] = W_K LN1(e[i] + pos[i]) + b_K,
+ * as the paper defines them (no rounding of the LN output; fp32 storage, double
+ * accumulation).  W_K [D][D]. */
 void orc_layer0_keys(const float* e, const float* pos, const float* ln_g, const float* ln_b,
                      const float* W_K, const float* b_K, int n, int D, float eps, float* k);
 /* One head: o[r] = softmax_j(<q[r], k[j]> / sqrt(dh)) v[j]; q [m][q_stride],

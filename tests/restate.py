@@ -77,11 +77,9 @@ def full(shape, W, frame):
 
 
 def layer0_keys(shape, W, e):
-    """Eq. 3 key vectors of every token: W_K bf16(LN1(e + pos)) + b_K (LN output rounded
-    to bf16 through float32, the precision the kernels take the decision in)."""
+    """Eq. 3 key vectors of every token in fp64: W_K LN1(e + pos) + b_K."""
     D = shape.dim
     xn = F.layer_norm(e + W["pos"], (D,), W["l0.ln1_g"], W["l0.ln1_b"], shape.ln_eps)
-    xn = xn.float().bfloat16().double()
     return F.linear(xn, W["l0.W_qkv"][D:2 * D], W["l0.b_qkv"][D:2 * D])
 
 
