@@ -102,7 +102,8 @@ int ivit_create(const ivit_config* cfg, const uint16_t* weights_bf16_host,
                 ivit_handle** out);
 
 /* Full encode of one frame per view (the paper's full forward that seeds the
- * reference, Sec. III-B).  frames_dev: uint8 [SV][img_h][img_w][3].
+ * reference, Sec. III-B).  frames_dev: uint8 [SV][img_h][img_w][3], any byte address
+ * (an odd address makes the patchify kernel use byte loads).
  * tokens_out_dev: bf16 [SV][N][D] final tokens (after the final LN), or NULL.
  * Re-seeds every cache and reference and marks every view warm. */
 int ivit_encode_full(ivit_handle* h, const uint8_t* frames_dev, uint16_t* tokens_out_dev,
@@ -177,9 +178,11 @@ void ivit_destroy(ivit_handle* h);
  *
  * It computes what the selection step of ivit_encode_incremental computes (cosine of
  * each token against its reference in fp32, then threshold or top-k), from embeddings
- * the caller holds: e_cur_dev and e_ref_dev fp32 [n_views][n_tok][dim].  Outputs, all
- * caller-owned device memory: idx_out_dev int32 [n_views][n_tok] (ascending updated
- * indices, then -1), counts_out_dev int32 [n_views].  Enqueued on `stream`; no handle.
+ * the caller holds: e_cur_dev and e_ref_dev fp32 [n_views][n_tok][dim], 16-byte
+ * aligned (they are read with 128-bit loads).  Outputs, all caller-owned device memory,
+ * 4-byte aligned: idx_out_dev int32 [n_views][n_tok] (ascending updated indices, then
+ * -1), counts_out_dev int32 [n_views].  A NULL or misaligned pointer returns
+ * IVIT_ERR_ARG before any device work.  Enqueued on `stream`; no handle.
  *
  * Its scratch (one fp32 score per token) is a file-scope device array of
  * IVIT_NOALLOC_MAX_TOKENS floats (256 KiB) that every GPU loading the library holds
@@ -187,7 +190,9 @@ void ivit_destroy(ivit_handle* h);
  * (message via ivit_last_error(NULL)); no cudaMalloc, cudaFree or allocating library
  * routine is ever called.  The first call on a device, with that device current, looks
  * up the array's device address (cudaGetSymbolAddress) and caches it: make that first
- * call before any stream capture.  All calls share the array; each call writes every
+ * call before any stream capture.  cudaDeviceReset invalidates the cached address:
+ * do not call this entry point on a device after resetting it in the same process.
+ * All calls share the array; each call writes every
  * score it reads, so nothing carries over, but calls that overlap on the GPU (two
  * streams, or two threads) race on it and must be serialised by the caller. */
 #define IVIT_NOALLOC_MAX_TOKENS 65536
@@ -202,8 +207,10 @@ int ivit_select_noalloc(const float* e_cur_dev, const float* e_ref_dev, int32_t 
  * memory; alpha, beta fp32 [batch]; b may be NULL, read as zero).  v0 and v7 are the
  * solver's anchor velocities (first and eighth step) and (alpha, beta, b) the adaptor's
  * prediction, all computed by the caller: this library holds neither network.  Needs no
- * handle; enqueued on `stream`, no allocation.  IVIT_ERR_ARG for negative sizes or a
- * NULL required pointer; batch * dim == 0 does nothing. */
+ * handle; enqueued on `stream`, no allocation.  IVIT_ERR_ARG for negative sizes, a
+ * NULL required pointer or a pointer that is not 4-byte aligned (checked before any
+ * device work); batch * dim == 0 does nothing.  128-bit accesses are used when dim is a
+ * multiple of 4 and the arrays are 16-byte aligned, scalar ones otherwise. */
 int ivit_action_combine(const float* x0_dev, const float* v0_dev, const float* v7_dev,
                         const float* alpha_dev, const float* beta_dev, const float* b_dev,
                         int32_t batch, int32_t dim, float* xT_dev, void* stream);

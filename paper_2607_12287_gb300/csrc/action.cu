@@ -14,11 +14,11 @@ namespace {
 __global__ void action_combine_kernel(const float* __restrict__ x0, const float* __restrict__ v0,
                                       const float* __restrict__ v7, const float* __restrict__ alpha,
                                       const float* __restrict__ beta, const float* __restrict__ b,
-                                      int dim, long long n, float* __restrict__ xT) {
+                                      int dim, long long n, int vec4, float* __restrict__ xT) {
   pdl_wait();
   pdl_launch_dependents();
   const long long stride = static_cast<long long>(gridDim.x) * blockDim.x;
-  if ((dim & 3) == 0) {
+  if (vec4) {
     const long long n4 = n >> 2;
     const float4* x4 = reinterpret_cast<const float4*>(x0);
     const float4* a4 = reinterpret_cast<const float4*>(v0);
@@ -51,14 +51,24 @@ extern "C" int ivit_action_combine(const float* x0_dev, const float* v0_dev, con
   const long long n = static_cast<long long>(batch) * dim;
   if (n == 0) return IVIT_OK;
   if (!x0_dev || !v0_dev || !v7_dev || !alpha_dev || !beta_dev || !xT_dev) return IVIT_ERR_ARG;
+  // 128-bit accesses need rows of a multiple of 4 floats and 16-byte aligned arrays;
+  // any other layout takes the scalar loop (alignment 4 bytes, checked here).
+  auto aligned = [](const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; };
+  for (const void* p : {static_cast<const void*>(x0_dev), static_cast<const void*>(v0_dev),
+                        static_cast<const void*>(v7_dev), static_cast<const void*>(alpha_dev),
+                        static_cast<const void*>(beta_dev), static_cast<const void*>(b_dev),
+                        static_cast<const void*>(xT_dev)})
+    if (p && !aligned(p, 4)) return IVIT_ERR_ARG;
+  const bool vec4 = (dim & 3) == 0 && aligned(x0_dev, 16) && aligned(v0_dev, 16) && aligned(v7_dev, 16) &&
+                    aligned(xT_dev, 16) && (!b_dev || aligned(b_dev, 16));
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev))
     return IVIT_ERR_CUDA;
-  const long long items = (dim & 3) == 0 ? n / 4 : n;
+  const long long items = vec4 ? n / 4 : n;
   const long long blocks = (items + 255) / 256;
   const int grid = static_cast<int>(blocks < 4LL * sms ? blocks : 4LL * sms);
   const cudaError_t e = ivit::launch_ex(ivit::action_combine_kernel, dim3(grid), dim3(256), 0,
                                         static_cast<cudaStream_t>(stream), 1, x0_dev, v0_dev, v7_dev, alpha_dev,
-                                        beta_dev, b_dev, static_cast<int>(dim), n, xT_dev);
+                                        beta_dev, b_dev, static_cast<int>(dim), n, vec4 ? 1 : 0, xT_dev);
   return e == cudaSuccess ? IVIT_OK : IVIT_ERR_CUDA;
 }

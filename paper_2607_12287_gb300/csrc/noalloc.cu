@@ -137,6 +137,13 @@ extern "C" int ivit_select_noalloc(const float* e_cur_dev, const float* e_ref_de
     ivit::set_create_error("ivit_select_noalloc: null pointer");
     return IVIT_ERR_ARG;
   }
+  // the score kernel reads both embedding sets with 128-bit loads, the selection kernel
+  // stores 32-bit indices: a misaligned pointer is an argument error, never a device fault
+  if ((reinterpret_cast<uintptr_t>(e_cur_dev) & 15u) || (reinterpret_cast<uintptr_t>(e_ref_dev) & 15u) ||
+      (reinterpret_cast<uintptr_t>(idx_out_dev) & 3u) || (reinterpret_cast<uintptr_t>(counts_out_dev) & 3u)) {
+    ivit::set_create_error("ivit_select_noalloc: e_cur/e_ref must be 16-byte aligned, idx/counts 4-byte aligned");
+    return IVIT_ERR_ARG;
+  }
   if (select_mode != IVIT_SEL_THRESHOLD && select_mode != IVIT_SEL_TOPK) {
     ivit::set_create_error("ivit_select_noalloc: bad select_mode");
     return IVIT_ERR_ARG;

@@ -28,10 +28,10 @@ __device__ __forceinline__ bool is_cold(const ColdMask& m, int v) {
 
 // --------------------------------------------------------------------- patchify
 // patches[v*N + i][(ky*P + kx)*3 + c] = frame[v][py*P + ky][px*P + kx][c] - 128 (exact in
-// bf16).  When a patch row (P*3 bytes) has even length, one thread per pair of adjacent
-// columns: 2 bytes in, one bf16 pair out, so consecutive threads read and write
-// contiguous runs; otherwise one thread per (token, ky) row.  Columns P*P*3 .. kpad-1
-// stay zero (set once at allocation).
+// bf16).  When a patch row (P*3 bytes) has even length and the frames start at an even
+// address, one thread per pair of adjacent columns: 2 bytes in, one bf16 pair out, so
+// consecutive threads read and write contiguous runs; otherwise one thread per (token,
+// ky) row with byte loads.  Columns P*P*3 .. kpad-1 stay zero (set once at allocation).
 __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __restrict__ patches,
                                 int sv, int img_h, int img_w, int P, int kpad) {
   pdl_wait();
@@ -39,7 +39,8 @@ __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __rest
   const int gw = img_w / P, gh = img_h / P, N = gw * gh;
   const int row = P * 3;
   const long long stride = static_cast<long long>(gridDim.x) * blockDim.x;
-  if ((row & 1) == 0 && static_cast<long long>(sv) * N * P * (row / 2) < (1LL << 30)) {
+  const bool even = (reinterpret_cast<uintptr_t>(frames) & 1u) == 0;
+  if ((row & 1) == 0 && even && static_cast<long long>(sv) * N * P * (row / 2) < (1LL << 30)) {
     // 32-bit index arithmetic (the divisions dominate this kernel's instruction count)
     const int pr = row / 2;  // column pairs per patch row
     const int total = sv * N * P * pr;

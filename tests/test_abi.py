@@ -136,3 +136,20 @@ def test_header_is_plain_c_and_links(pkg, tmp_path):
     code, null_out, msg = out[1].split(" ", 2)
     assert int(code) == pkg.IVIT_ERR_SHAPE and null_out == "1" and "64" in msg
     assert int(out[2]) == pkg.IVIT_ERR_ARG
+
+
+def test_misaligned_pointers_rejected_before_device_work(pkg):
+    # raw addresses: the entry points must turn a misaligned pointer into IVIT_ERR_ARG
+    # on the host, before any CUDA call (none can succeed on a machine without a GPU)
+    L = pkg.load()
+    ok16, off4, odd = 0x10000, 0x10004, 0x10001
+    assert L.ivit_select_noalloc(off4, ok16, 1, 16, 8, 0, 0.98, 0, ok16, ok16, None) == pkg.IVIT_ERR_ARG
+    assert L.ivit_select_noalloc(ok16, off4, 1, 16, 8, 0, 0.98, 0, ok16, ok16, None) == pkg.IVIT_ERR_ARG
+    assert L.ivit_select_noalloc(ok16, ok16, 1, 16, 8, 0, 0.98, 0, odd, ok16, None) == pkg.IVIT_ERR_ARG
+    assert L.ivit_select_noalloc(ok16, ok16, 1, 16, 8, 0, 0.98, 0, ok16, odd, None) == pkg.IVIT_ERR_ARG
+    assert "aligned" in pkg.ivit_last_error(None)
+    for i in range(7):
+        ptrs = [ok16] * 7
+        ptrs[i] = odd
+        x0, v0, v7, al, be, b, xT = ptrs
+        assert L.ivit_action_combine(x0, v0, v7, al, be, b, 2, 8, xT, None) == pkg.IVIT_ERR_ARG

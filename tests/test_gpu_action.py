@@ -34,3 +34,25 @@ def test_action_combine_empty_and_bad_args(pkg):
     lib = pkg.load()
     assert lib.ivit_action_combine(None, None, None, None, None, None, 2, 3, None, None) == pkg.IVIT_ERR_ARG
     assert lib.ivit_action_combine(None, None, None, None, None, None, -1, 3, None, None) == pkg.IVIT_ERR_ARG
+
+
+def test_action_combine_offset_views_take_the_scalar_path(pkg, oracle_mod):
+    # views starting 4 bytes into their storage are not 16-byte aligned: the library must
+    # fall back to scalar accesses instead of faulting on 128-bit ones
+    import torch
+    B, A = 6, 64
+    rng = np.random.Generator(np.random.PCG64(7))
+    x0, v0, v7, b = (rng.standard_normal((B, A)).astype(np.float32) for _ in range(4))
+    al, be = (rng.standard_normal(B).astype(np.float32) for _ in range(2))
+    want = oracle_mod.action_combine(x0, v0, v7, al, be, b)
+
+    def off(a):
+        t = torch.zeros(a.size + 1, dtype=torch.float32, device="cuda")
+        t[1:] = torch.from_numpy(a.ravel()).cuda()
+        return t[1:].view(a.shape)
+
+    outb = torch.full((B * A + 1,), float("nan"), dtype=torch.float32, device="cuda")
+    out = outb[1:].view(B, A)
+    assert out.data_ptr() % 16 == 4
+    pkg.ivit_action_combine(off(x0), off(v0), off(v7), off(al), off(be), off(b), out)
+    np.testing.assert_allclose(out.cpu().numpy(), want, rtol=2e-6, atol=2e-6)

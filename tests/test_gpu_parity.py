@@ -233,3 +233,31 @@ def test_many_keys_online_softmax_groups(pkg, oracle_mod):
     w = synth.make_weights(shape, 131)
     frames = list(synth.stream_random(shape, 32, 3, 132, change_p=0.15))
     run_side_by_side(pkg, oracle_mod, shape, w, frames, 16, 2, check_caches=True)
+
+
+def test_frames_at_an_odd_address(pkg, monkeypatch):
+    # without graphs the patchify kernel reads the caller's frames directly: frames that
+    # start at an odd byte address take its byte-load path and must give the same tokens
+    import torch
+    monkeypatch.setenv("IVIT_NO_GRAPH", "1")
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 141)
+    f0, f1 = synth.stream_random(shape, 2, 2, 142, change_p=0.3)
+    outs = []
+    for odd in (False, True):
+        enc = pkg.IncrementalViT(shape, w, 1, 2)
+        try:
+            got = []
+            for f in (f0, f1):
+                buf = torch.zeros(f.size + 1, dtype=torch.uint8, device="cuda")
+                fd = buf[1:] if odd else buf[:-1]
+                fd.copy_(torch.from_numpy(f).reshape(-1).cuda())
+                fd = fd.view(f.shape)
+                assert (fd.data_ptr() % 2 == 1) == odd
+                got.append(enc.encode_full(fd) if not got else enc.encode_incremental(fd)[0])
+            outs.append([g.clone() for g in got])
+            assert enc.device_status() == 0
+        finally:
+            enc.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)

@@ -54,6 +54,54 @@ def test_noalloc_selection_matches_encoder(pkg, mode, k):
         enc.close()
 
 
+@pytest.mark.parametrize("mode,k", [(synth.SEL_THRESHOLD, 0), (synth.SEL_TOPK, 11)])
+def test_noalloc_selection_matches_oracle(pkg, oracle_mod, mode, k):
+    """The lists against the oracle's selection (Eq. 3 cosine in fp32 with double sums,
+    then the threshold or top-k of Sec. III-B) on the same embeddings, two calls in a
+    row; the oracle's scores keep a margin from every decision boundary."""
+    import torch
+    V, N, D = 4, 196, 192
+    rng = np.random.Generator(np.random.PCG64(31 + k))
+    cur = rng.standard_normal((V, N, D)).astype(np.float32)
+    for call in range(2):
+        ref = cur.copy()
+        # a fifth of the tokens change a lot, the rest by a little noise
+        moved = rng.random((V, N)) < 0.2
+        cur = ref + np.where(moved[..., None], 0.9, 0.01) * rng.standard_normal((V, N, D)).astype(np.float32)
+        idx = torch.full((V, N), -7, dtype=torch.int32, device="cuda")
+        cnt = torch.full((V,), -7, dtype=torch.int32, device="cuda")
+        pkg.ivit_select_noalloc(torch.from_numpy(cur).cuda(), torch.from_numpy(ref).cuda(), V, N, D, mode,
+                                0.98, k, idx, cnt)
+        torch.cuda.synchronize()
+        for v in range(V):
+            sims = np.array([oracle_mod.cosine(cur[v, i], ref[v, i]) for i in range(N)], np.float32)
+            if mode == synth.SEL_THRESHOLD:
+                assert np.abs(sims - 0.98).min() > 1e-3
+                want = oracle_mod.select_threshold(sims, 0.98)
+            else:
+                srt = np.sort(sims)
+                assert srt[k] - srt[k - 1] > 1e-4
+                want = oracle_mod.select_topk(sims, k)
+            assert int(cnt[v]) == len(want), f"call {call} view {v}"
+            got = idx[v].cpu().numpy()
+            np.testing.assert_array_equal(got[:len(want)], want)
+            assert np.all(got[len(want):] == -1)
+
+
+def test_noalloc_rejects_misaligned_views(pkg):
+    import torch
+    V, N, D = 1, 16, 8
+    buf = torch.zeros(V * N * D + 1, dtype=torch.float32, device="cuda")
+    ok = buf[:-1]
+    off = buf[1:]  # starts 4 bytes into the allocation: not 16-byte aligned
+    ib = torch.zeros(V * N, dtype=torch.int32, device="cuda")
+    cb = torch.zeros(V, dtype=torch.int32, device="cuda")
+    for a, b in ((off, ok), (ok, off)):
+        with pytest.raises(pkg.IvitError) as e:
+            pkg.ivit_select_noalloc(a, b, V, N, D, 0, 0.98, 0, ib, cb)
+        assert e.value.code == pkg.IVIT_ERR_ARG
+
+
 def test_noalloc_rejects_oversize(pkg):
     import torch
     buf = torch.zeros(8, dtype=torch.float32, device="cuda")
