@@ -31,9 +31,12 @@ def assert_tokens_close(gpu: np.ndarray, ref: np.ndarray, what: str = ""):
 
 def run_side_by_side(pkg, oracle_mod, shape, weights, frames, n_streams=1, n_views=1,
                      select_mode=0, threshold=0.98, topk=0, ref_mode=0, margin=2e-3,
-                     check_caches=False, first_full=True, score_source=0, schedule=0, mlp_tokens=0):
+                     check_caches=False, first_full=True, score_source=0, schedule=0, mlp_tokens=0,
+                     cache_layers="ends"):
     """Feeds ``frames`` (list of uint8 [SV,H,W,3]) to both sides; frame 0 is a full
-    encode when ``first_full``.  Returns per-frame (rel, cos, counts)."""
+    encode when ``first_full``.  With ``check_caches`` the per-layer caches of the first
+    and last layer (``cache_layers="ends"``) or of every layer (``"all"``) are compared
+    after the last frame.  Returns per-frame (rel, cos, counts)."""
     import torch
 
     enc = pkg.IncrementalViT(shape, weights, n_streams, n_views, select_mode, threshold, topk,
@@ -70,7 +73,8 @@ def run_side_by_side(pkg, oracle_mod, shape, weights, frames, n_streams=1, n_vie
             rel, cos = assert_tokens_close(got, ref, f"frame {t}")
             stats.append((rel, cos, counts))
         if check_caches:
-            for l in (0, shape.depth - 1):
+            layers = range(shape.depth) if cache_layers == "all" else sorted({0, shape.depth - 1})
+            for l in layers:
                 for which in ("K", "V", "A") if mlp_tokens else ("K", "V"):
                     g = enc.cache(which, l).float().cpu().numpy()
                     r = orc.cache(which, l)
