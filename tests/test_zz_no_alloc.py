@@ -67,7 +67,8 @@ def test_noalloc_selection_matches_oracle(pkg, oracle_mod, mode, k):
         ref = cur.copy()
         # a fifth of the tokens change a lot, the rest by a little noise
         moved = rng.random((V, N)) < 0.2
-        cur = ref + np.where(moved[..., None], 0.9, 0.01) * rng.standard_normal((V, N, D)).astype(np.float32)
+        step = np.where(moved[..., None], 0.9, 0.01) * rng.standard_normal((V, N, D))
+        cur = (ref + step).astype(np.float32)
         idx = torch.full((V, N), -7, dtype=torch.int32, device="cuda")
         cnt = torch.full((V,), -7, dtype=torch.int32, device="cuda")
         pkg.ivit_select_noalloc(torch.from_numpy(cur).cuda(), torch.from_numpy(ref).cuda(), V, N, D, mode,
