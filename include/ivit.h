@@ -154,12 +154,15 @@ int ivit_profile_read(ivit_handle* h, double* gemm_ms_total, int64_t* gemm_launc
  * wait expired, the kernel skipped its work and returned).  Synchronises `stream`. */
 int ivit_device_status(ivit_handle* h, void* stream);
 
-/* Execution paths (chosen at create; the environment variable IVIT_PATH=kernels or
- * IVIT_PATH=persistent selects one for every call): one kernel per operation, chained
- * with programmatic dependent launch and replayed as a CUDA graph (every incremental
- * call, and the full encodes for dim > 384), or every transformer block of a call in
- * one persistent cooperative kernel with grid barriers (the full encodes for
- * dim <= 384, where per-operation launches dominate).  Both give the same result. */
+/* Execution paths (chosen at create; the environment variable IVIT_PATH=kernels,
+ * IVIT_PATH=persistent or IVIT_PATH=stream selects one): one kernel per operation,
+ * chained with programmatic dependent launch and replayed as a CUDA graph (every
+ * incremental call, and the full encodes for dim > 384); every transformer block of a
+ * call in one persistent cooperative kernel with grid barriers (the full encodes for
+ * dim <= 384, where per-operation launches dominate); or, on request only
+ * (IVIT_PATH=stream), the incremental calls without cold views in one cooperative
+ * weight-streaming kernel that keeps each SM's share of the next weights in flight
+ * through a shared-memory ring.  All give the same result within the bf16 rounding. */
 
 /* Number of the library's kernel launches made by the last encode call. */
 int64_t ivit_last_launch_count(const ivit_handle* h);

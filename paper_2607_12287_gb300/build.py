@@ -15,7 +15,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libivit.so")
-SOURCES = ["gemm.cu", "ops.cu", "attention.cu", "persistent.cu", "engine.cu", "noalloc.cu", "action.cu"]
+SOURCES = ["gemm.cu", "ops.cu", "attention.cu", "persistent.cu", "stream.cu", "engine.cu", "noalloc.cu",
+           "action.cu"]
 HEADERS = ["ptx.cuh", "internal.h"]
 NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

@@ -144,6 +144,15 @@ struct ivit_handle {
   void* pt_mem = nullptr;  // device: tensor maps, layer parameters, partials, barrier words
   ivit::PersistentArgs pt_args{};
 
+  // Weight-streaming kernel (every block of an incremental call in one cooperative
+  // launch, weights streamed through a shared-memory ring) for small updated-row counts.
+  bool stream_ok = false;
+  size_t sk_smem = 0;
+  int sk_grid = 0;
+  void* sk_mem = nullptr;  // device: tensor maps, layer parameters, partials, sync words
+  size_t sk_sync_bytes = 0;
+  ivit::StreamArgs sk_args{};
+
   // CUDA graphs of the full and the steady-state incremental chain.  Inputs and outputs
   // are staged through handle-owned buffers (copies outside the graph), so the graph's
   // kernel parameters never change.
@@ -330,6 +339,119 @@ int setup_persistent(ivit_handle* h) {
   h->pt_grid = grid;
   h->persistent = true;
   h->persistent_inc = forced;
+  return IVIT_OK;
+}
+
+// Prepares the weight-streaming kernel (IVIT_PATH=stream: every incremental call without
+// a cold view runs it).  It is not the default: on the So400m camera stream it measured
+// 1.5 ms per frame against the kernel chain's 1.0 ms (seven grid barriers per layer and
+// the dependent latencies inside each stage cost more than the chain's launch handoffs).
+int setup_stream(ivit_handle* h) {
+  const ivit_config& c = h->cfg;
+  const char* path = std::getenv("IVIT_PATH");
+  if (!path || std::strcmp(path, "stream") != 0) return IVIT_OK;
+  if (c.mlp_tokens == IVIT_MLP_ALL) return IVIT_OK;  // the kernel chain runs that reading
+  const int N = h->N, D = h->D, F = h->F, H = h->H, L = h->L, SV = h->SV, dh = D / H;
+  if (D > ivit::stream_max_dim() || N > 256) return IVIT_OK;
+  int optin = 0;
+  IVIT_CK(h, cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, h->device));
+  const int grid = h->num_sms;
+  // K splits: enough tasks (tile x split) to give about one to every CTA
+  const int n_out[4] = {3 * D, D, F, D}, kdim[4] = {D, D, D, F};
+  int splits[4], max_kb = 0;
+  size_t part_floats = 0;
+  for (int g = 0; g < 4; ++g) {
+    const int tiles = (n_out[g] + 127) / 128, nkb = (kdim[g] + 63) / 64;
+    splits[g] = std::max(1, std::min(nkb, grid / tiles));
+    max_kb = std::max(max_kb, ivit::stream_task_kblocks(kdim[g], splits[g]));
+    part_floats = std::max(part_floats, static_cast<size_t>(splits[g]) * h->M_max * n_out[g]);
+  }
+  const size_t region = ivit::stream_region_bytes(max_kb, N, dh);
+  const int rs = ivit::stream_ring_stages_for(static_cast<size_t>(optin), region);
+  if (rs < std::max(4, max_kb)) return IVIT_OK;
+  const size_t smem = ivit::stream_smem_bytes(rs, region);
+  IVIT_CK(h, ivit::stream_setup(smem));
+  if (ivit::stream_max_ctas(smem) < grid) return IVIT_OK;
+  const int rpp = ivit::stream_rows_per_pass();
+  const int passes_max = (h->M_max + rpp - 1) / rpp;
+  const int qkv_tiles = (3 * D + 127) / 128, up_tiles = (F + 127) / 128;
+  const size_t sync_words = 4 + static_cast<size_t>(L) * (qkv_tiles + up_tiles) * passes_max;
+  Arena ka;
+  const size_t o_w = ka.take(sizeof(CUtensorMap) * 4 * L), o_b = ka.take(sizeof(CUtensorMap) * 3);
+  const size_t o_kv = ka.take(sizeof(CUtensorMap) * 2 * L), o_lp = ka.take(sizeof(ivit::LayerParams) * L);
+  const size_t o_part = ka.take(part_floats * sizeof(float)), o_sync = ka.take(sync_words * sizeof(unsigned));
+  IVIT_CK(h, cudaMalloc(&h->sk_mem, ka.size));
+  IVIT_CK(h, cudaMemset(h->sk_mem, 0, ka.size));
+  ka.base = static_cast<char*>(h->sk_mem);
+  std::vector<CUtensorMap> wm(4 * L), kvm(2 * L);
+  std::vector<ivit::LayerParams> lp(L);
+  for (int l = 0; l < L; ++l) {
+    const LayerW& w = h->layers[l];
+    const size_t off = static_cast<size_t>(l) * h->M_max * D;
+    wm[4 * l + 0] = w.tm_qkv;
+    wm[4 * l + 1] = w.tm_o;
+    wm[4 * l + 2] = w.tm_1;
+    wm[4 * l + 3] = w.tm_2;
+    if (!make_map(&kvm[2 * l], h->cacheK + off, D, h->M_max, D * 2, dh, N, false) ||
+        !make_map(&kvm[2 * l + 1], h->cacheV + off, D, h->M_max, D * 2, dh, N, false))
+      return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for the weight-streaming kernel");
+    lp[l] = ivit::LayerParams{w.bqkv, w.bo, w.b1, w.b2, w.ln1g, w.ln1b, w.ln2g, w.ln2b};
+  }
+  const CUtensorMap bm[3] = {h->tm_xn, h->tm_o, h->tm_h};
+  IVIT_CK(h, cudaMemcpy(ka.base + o_w, wm.data(), sizeof(CUtensorMap) * 4 * L, cudaMemcpyHostToDevice));
+  IVIT_CK(h, cudaMemcpy(ka.base + o_b, bm, sizeof(bm), cudaMemcpyHostToDevice));
+  IVIT_CK(h, cudaMemcpy(ka.base + o_kv, kvm.data(), sizeof(CUtensorMap) * 2 * L, cudaMemcpyHostToDevice));
+  IVIT_CK(h, cudaMemcpy(ka.base + o_lp, lp.data(), sizeof(ivit::LayerParams) * L, cudaMemcpyHostToDevice));
+  ivit::StreamArgs& a = h->sk_args;
+  a.N = N;
+  a.D = D;
+  a.F = F;
+  a.H = H;
+  a.dh = dh;
+  a.L = L;
+  a.SV = SV;
+  a.M_max = h->M_max;
+  a.eps = c.ln_eps;
+  a.gelu = c.gelu;
+  a.ring_stages = rs;
+  a.region_bytes = static_cast<int>(region);
+  a.att_groups = std::max(1, std::min(16, grid / std::max(1, SV * H)));
+  for (int g = 0; g < 4; ++g) a.splits[g] = splits[g];
+  a.qkv_tiles = qkv_tiles;
+  a.n_barriers = 7 * L;
+  a.cu_rows = h->cu_rows;
+  a.rowtok = h->rowtok;
+  a.wmaps = ka.at<CUtensorMap>(o_w);
+  a.bmaps = ka.at<CUtensorMap>(o_b);
+  a.kvmaps = ka.at<CUtensorMap>(o_kv);
+  a.layers = ka.at<ivit::LayerParams>(o_lp);
+  a.lnfg = h->lnfg;
+  a.lnfb = h->lnfb;
+  a.x = h->x;
+  a.xn = h->xn;
+  a.q = h->q;
+  a.o = h->o;
+  a.h = h->hbuf;
+  a.cacheK = h->cacheK;
+  a.cacheV = h->cacheV;
+  a.tok_out = h->tok_out;
+  a.part = ka.at<float>(o_part);
+  a.sync = ka.at<unsigned>(o_sync);
+  a.err = h->err;
+  a.trace = nullptr;
+  if (std::getenv("IVIT_TRACE")) {
+    const size_t n = static_cast<size_t>(a.n_barriers) * (grid + 1) + 64 * static_cast<size_t>(grid);
+    IVIT_CK(h, cudaMalloc(&a.trace, n * sizeof(unsigned long long)));
+    IVIT_CK(h, cudaMemset(a.trace, 0, n * sizeof(unsigned long long)));
+  }
+  h->sk_sync_bytes = sync_words * sizeof(unsigned);
+  h->sk_smem = smem;
+  h->sk_grid = grid;
+  h->stream_ok = true;
+  if (std::getenv("IVIT_DEBUG"))
+    std::fprintf(stderr, "ivit stream kernel: grid %d, smem %zu, ring %d stages, region %zu, groups %d, "
+                 "splits %d %d %d %d\n", grid, smem, rs, region, a.att_groups, splits[0], splits[1], splits[2],
+                 splits[3]);
   return IVIT_OK;
 }
 
@@ -556,11 +678,16 @@ int setup(ivit_handle* h, const uint16_t* wb) {
       !make_map(&h->tm_h, h->hbuf, F, M, F * 2, 64, 32))
     return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
   if (int r = setup_persistent(h)) return r;
+  if (int r = setup_stream(h)) return r;
   IVIT_CK(h, cudaDeviceSynchronize());
   return IVIT_OK;
 }
 
 void release(ivit_handle* h) {
+  if (h->sk_args.trace) cudaFree(h->sk_args.trace);
+  h->sk_args.trace = nullptr;
+  if (h->sk_mem) cudaFree(h->sk_mem);
+  h->sk_mem = nullptr;
   if (h->pt_args.trace) cudaFree(h->pt_args.trace);
   h->pt_args.trace = nullptr;
   if (h->pt_mem) cudaFree(h->pt_mem);
@@ -632,6 +759,64 @@ void print_trace(ivit_handle* h, cudaStream_t s) {
                1e-3 * static_cast<double>(t[n] - t[1]), 1e-3 * static_cast<double>(t[2] - t[1]));
   for (int k = 0; k < 9; ++k)
     if (cnt[k]) std::fprintf(stderr, "  %-12s %6.2f us x %d\n", names[k], acc[k] / cnt[k], cnt[k]);
+}
+
+// Debug aid (IVIT_TRACE): stage durations of the last weight-streaming launch (critical
+// path: the last CTA's arrival at each grid barrier after the previous barrier's exit),
+// barrier latencies, and per-task phase times.
+void print_stream_trace(ivit_handle* h, cudaStream_t s) {
+  const int L = h->L, G = h->sk_grid, NB = h->sk_args.n_barriers;
+  std::vector<unsigned long long> t(static_cast<size_t>(NB) * (G + 1) + 64 * static_cast<size_t>(G));
+  if (cudaStreamSynchronize(s) != cudaSuccess) return;
+  cudaMemcpy(t.data(), h->sk_args.trace, t.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost);
+  static const char* names[7] = {"qkv", "attention", "out", "ln2", "up", "down", "ln1"};
+  double dur[7] = {0}, lat[7] = {0}, mean_arr[7] = {0};
+  int cnt[7] = {0};
+  for (int k = 1; k < NB; ++k) {
+    unsigned long long mx = 0;
+    double sum = 0;
+    for (int c = 0; c < G; ++c) {
+      mx = std::max(mx, t[static_cast<size_t>(k) * G + c]);
+      sum += static_cast<double>(t[static_cast<size_t>(k) * G + c]);
+    }
+    const double prev_exit = static_cast<double>(t[static_cast<size_t>(NB) * G + k - 1]);
+    const double exit_k = static_cast<double>(t[static_cast<size_t>(NB) * G + k]);
+    const int j = (k - 1) % 7;
+    dur[j] += 1e-3 * (static_cast<double>(mx) - prev_exit);
+    lat[j] += 1e-3 * (exit_k - static_cast<double>(mx));
+    mean_arr[j] += 1e-3 * (sum / G - prev_exit);
+    ++cnt[j];
+  }
+  std::fprintf(stderr, "ivit stream trace: %d barriers, first exit %.1f us after CTA 0 arrived, last exit %.1f us\n",
+               NB, 1e-3 * static_cast<double>(t[static_cast<size_t>(NB) * G] - t[0]),
+               1e-3 * static_cast<double>(t[static_cast<size_t>(NB) * G + NB - 1] - t[0]));
+  for (int j = 0; j < 7; ++j)
+    if (cnt[j])
+      std::fprintf(stderr, "  %-9s stage %6.2f us (mean arrival %6.2f) barrier %5.2f us\n", names[j], dur[j] / cnt[j],
+                   mean_arr[j] / cnt[j], lat[j] / cnt[j]);
+  static const char* kinds[6] = {"qkv", "out", "up", "down", "attn", "rows"};
+  static const char* slots[6][7] = {{"w-wait", "B", "mma", "acc-wait", "epilogue", "fixup", ""},
+                                    {"w-wait", "B", "mma", "acc-wait", "epilogue", "fixup", ""},
+                                    {"w-wait", "B", "mma", "acc-wait", "epilogue", "fixup", ""},
+                                    {"w-wait", "B", "mma", "acc-wait", "epilogue", "fixup", ""},
+                                    {"kv+patch", "compute", "scores", "softmax+pv", "", "", ""},
+                                    {"row", "", "", "", "", "", ""}};
+  const size_t base = static_cast<size_t>(NB) * (G + 1);
+  for (int g = 0; g < 6; ++g) {
+    double n = 0;
+    for (int c = 0; c < G; ++c) n += static_cast<double>(t[base + (c * 8 + g) * 8 + 7]);
+    if (n == 0) continue;
+    std::fprintf(stderr, "  %-5s x%6.0f/call:", kinds[g], n);
+    for (int k = 0; k < 7; ++k) {
+      if (!slots[g][k][0]) continue;
+      double sum = 0;
+      for (int c = 0; c < G; ++c) sum += 1e-3 * static_cast<double>(t[base + (c * 8 + g) * 8 + k]);
+      std::fprintf(stderr, " %s %.2f", slots[g][k], sum / n);
+    }
+    std::fprintf(stderr, "\n");
+  }
+  (void)L;
+  cudaMemset(h->sk_args.trace, 0, t.size() * sizeof(unsigned long long));
 }
 
 // Attention of the updated queries over all tokens of their view for one layer.
@@ -811,6 +996,19 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
                                  c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
   ++h->launches;
 
+  bool any_cold = false;
+  for (int v = 0; v < SV; ++v) any_cold = any_cold || (cm.bits[v >> 5] >> (v & 31)) & 1u;
+  if (h->stream_ok && !full && !any_cold) {
+    IVIT_CK(h, cudaMemsetAsync(h->sk_args.sync, 0, h->sk_sync_bytes, s));
+    IVIT_CK(h, ivit::launch_stream(h->sk_args, h->sk_grid, h->sk_smem, s));
+    ++h->launches;
+    if (h->sk_args.trace) {
+      cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+      cudaStreamIsCapturing(s, &cs);
+      if (cs == cudaStreamCaptureStatusNone) print_stream_trace(h, s);
+    }
+    return IVIT_OK;
+  }
   if (h->persistent && (full || h->persistent_inc)) {
     IVIT_CK(h, cudaMemsetAsync(h->pt_args.gbar, 0, 4 * sizeof(unsigned), s));
     IVIT_CK(h, ivit::launch_persistent(h->pt_args, h->pt_grid, h->pt_smem, s));

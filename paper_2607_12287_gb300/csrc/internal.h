@@ -123,6 +123,52 @@ int persistent_max_ctas(size_t smem);
 // Cooperative launch (all CTAs resident); fails if the grid cannot be resident.
 cudaError_t launch_persistent(const PersistentArgs& a, int grid, size_t smem, cudaStream_t s);
 
+// ------------------------------------------------ weight-streaming encoder (small M)
+struct StreamArgs {
+  int N, D, F, H, dh, L, SV, M_max;
+  float eps;
+  int gelu;
+  int ring_stages;                // weight ring depth (16 KB stages), >= the k-blocks of a task
+  int region_bytes;               // activation operand / attention region of shared memory
+  int att_groups;                 // query groups per (view, head)
+  int splits[4];                  // K splits of the QKV, out-proj, MLP-up and MLP-down GEMMs
+  int qkv_tiles;                  // 128-feature tiles of the QKV GEMM
+  int n_barriers;                 // grid barriers per launch (7 L)
+  const int* cu_rows;             // [SV+1], cu_rows[SV] = updated rows M
+  const int* rowtok;              // [M] packed row -> token v*N + i
+  const CUtensorMap* wmaps;       // [L][4] weights (qkv, out, up, down), box 64 x 128, 128B swizzle
+  const CUtensorMap* bmaps;       // [3] LN output xn, attention output o, MLP hidden h; box 64 x 32
+  const CUtensorMap* kvmaps;      // [L][2] key / value caches, box dh x N, no swizzle
+  const LayerParams* layers;      // [L], device memory
+  const float *lnfg, *lnfb;
+  float* x;                       // fp32 residual stream [M_max][D] (packed rows)
+  bf16 *xn, *q, *o, *h, *cacheK, *cacheV, *tok_out;
+  float* part;                    // split partials [splits][M_max][n_out] of the current GEMM
+  unsigned* sync;                 // [0] barrier count, [2] abort, [4 + ...] tile counters of the
+                                  // QKV and MLP-up GEMMs [L][tiles][passes]; zeroed per launch
+  int* err;
+  // Optional timeline (IVIT_TRACE): [n_barriers][G] barrier arrival times,
+  // [n_barriers] barrier exit times of CTA 0, [G][8][8] per-CTA accumulators.
+  unsigned long long* trace;
+};
+
+// k-blocks (64 wide) of one task of a GEMM with K = k split `splits` ways.
+int stream_task_kblocks(int k, int splits);
+// Bytes of the activation operand / attention region (1 KB multiple).
+size_t stream_region_bytes(int max_task_kblocks, int n_tok, int head_dim);
+// Dynamic shared memory of one CTA with `ring_stages` 16 KB weight stages.
+size_t stream_smem_bytes(int ring_stages, size_t region);
+// Most weight stages that fit beside the region within `smem_limit` bytes (<= 16).
+int stream_ring_stages_for(size_t smem_limit, size_t region);
+// Largest model width a row stage holds in registers.
+int stream_max_dim();
+// Updated rows per pass of a GEMM task.
+int stream_rows_per_pass();
+cudaError_t stream_setup(size_t smem);
+int stream_max_ctas(size_t smem);
+// Cooperative launch (all CTAs resident); fails if the grid cannot be resident.
+cudaError_t launch_stream(const StreamArgs& a, int grid, size_t smem, cudaStream_t s);
+
 // ------------------------------------------------------------------- other kernels
 struct ColdMask {
   uint32_t bits[128];  // bit v set: view v is cold (updates every token); up to 4096 views

@@ -135,18 +135,19 @@ def forced_path(request, monkeypatch):
     return request.param
 
 
-@pytest.mark.parametrize("forced_path", ["kernels", "persistent"], indirect=True)
+@pytest.mark.parametrize("forced_path", ["kernels", "persistent", "stream"], indirect=True)
 @pytest.mark.parametrize("shape,S,V", [(SHAPE_A, 1, 3), (SHAPE_C, 1, 2)], ids=["A", "C"])
 def test_both_execution_paths(pkg, oracle_mod, forced_path, shape, S, V):
-    # the per-operation kernel chain and the persistent all-layers kernel give the same
-    # lists and tokens within tolerance (full encode, cold start and steady state)
+    # the per-operation kernel chain, the persistent all-layers kernel and the
+    # weight-streaming kernel give the same lists and tokens within tolerance (full
+    # encode, cold start and steady state)
     w = synth.make_weights(shape, 25)
     frames = list(synth.stream_random(shape, S * V, 4, 26, change_p=0.15))
     run_side_by_side(pkg, oracle_mod, shape, w, frames, S, V, check_caches=True)
     run_side_by_side(pkg, oracle_mod, shape, w, frames[:2], S, V, first_full=False)
 
 
-@pytest.mark.parametrize("forced_path", ["kernels", "persistent"], indirect=True)
+@pytest.mark.parametrize("forced_path", ["kernels", "persistent", "stream"], indirect=True)
 @pytest.mark.parametrize("mode,k", [(synth.SEL_THRESHOLD, 0), (synth.SEL_TOPK, 11)])
 def test_first_layer_key_scores(pkg, oracle_mod, forced_path, mode, k):
     # Eq. 3 as printed: cosine of the first layer's keys of every token.  Top-k repaints
@@ -261,3 +262,17 @@ def test_frames_at_an_odd_address(pkg, monkeypatch):
             enc.close()
     for a, b in zip(*outs):
         assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("forced_path", ["stream"], indirect=True)
+@pytest.mark.parametrize("p", [0.1, 0.3])
+def test_stream_kernel_row_passes(pkg, oracle_mod, forced_path, p):
+    # 2 streams of 196 tokens: about 39 and 118 updated rows per call, so the
+    # weight-streaming kernel runs its rows in 2 to 4 passes of 32 (weights kept in the
+    # ring across passes, the MLP-down split partials of every pass summed by the last
+    # split); erf GELU, a ragged MLP width (768 = 24 slices) and several attention groups
+    shape = SHAPE_B
+    w = synth.make_weights(shape, 151)
+    frames = list(synth.stream_random(shape, 2, 4, 152, change_p=p))
+    stats = run_side_by_side(pkg, oracle_mod, shape, w, frames, 2, 1, check_caches=True)
+    assert max(int(st[2].sum()) for st in stats[1:]) > 32

@@ -112,6 +112,14 @@ def test_so400m_448_batched_every_view_two_layers(pkg, oracle_mod):
     assert all(s[2].min() > 0 for s in stats[1:])
 
 
+def test_so400m_1view_prefix_stream_path(pkg, oracle_mod, monkeypatch):
+    # the opt-in weight-streaming kernel at full size (every layer's caches compared)
+    monkeypatch.setenv("IVIT_PATH", "stream")
+    wl = synth.WORKLOADS["so400m_224_1view"]
+    w = synth.make_weights(wl.shape, 0)
+    run_side_by_side(pkg, oracle_mod, wl.shape, w, _frames(wl, 4), check_caches=True, cache_layers="all")
+
+
 def test_so400m_1view_prefix_persistent_path(pkg, oracle_mod, monkeypatch):
     monkeypatch.setenv("IVIT_PATH", "persistent")
     wl = synth.WORKLOADS["so400m_224_1view"]
