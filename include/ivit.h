@@ -143,12 +143,21 @@ int ivit_get_cache(ivit_handle* h, int which, int layer, void* dst_dev, void* st
  * IVIT_ERR_ARG if stream_index is outside [-1, n_streams). */
 int ivit_reset(ivit_handle* h, int stream_index);
 
-/* Kernel timing hook: when enabled, every launch of the dominant kernel family (the
- * tensor-core GEMM) is bracketed by CUDA events on the launch stream; the sum and
- * count since the last call are returned and reset. */
-int ivit_profile_enable(ivit_handle* h, int enable);
-int ivit_profile_read(ivit_handle* h, double* gemm_ms_total, int64_t* gemm_launches,
-                      double* gemm_bytes_total);
+/* Kernel timeline.  With enable != 0 every later call records, for each of its kernel
+ * launches, the global time at which each CTA started its work (after the wait on the
+ * previous kernel) and finished; the captured CUDA graphs are rebuilt with the
+ * recording in them, so the calls still run as replayed graphs (enable = 0 rebuilds
+ * them without it).  Allocates 8 MB of device memory on first use.
+ * ivit_timeline_read synchronises `stream` and reads the last call: per kernel family
+ * (index 0 tensor-core GEMMs, 1 attention, 2 layer norms, 3 patchify / score /
+ * selection / gather) the sum over its launches of (last CTA end - first CTA start)
+ * in ms and the number of launches (arrays of 4, either may be NULL), the algorithmic
+ * bytes of the GEMM launches (weights + input rows + outputs + bias, with this call's
+ * updated-row count), and the span from the first start to the last end in ms.  Only
+ * the first 1024 CTAs of a launch record.  IVIT_ERR_ARG when timeline mode is off. */
+int ivit_timeline(ivit_handle* h, int enable);
+int ivit_timeline_read(ivit_handle* h, void* stream, double* family_ms, int64_t* family_launches,
+                       double* gemm_bytes_total, double* span_ms);
 
 /* Reads and clears the device error word (0 = none; nonzero = a kernel's bounded
  * wait expired, the kernel skipped its work and returned).  Synchronises `stream`. */

@@ -27,8 +27,8 @@ IVIT_ERR_DEVICE = -5
 
 EXPORTED = [
     "ivit_weights_size", "ivit_create", "ivit_encode_full", "ivit_encode_incremental",
-    "ivit_get_changed", "ivit_get_cache", "ivit_reset", "ivit_profile_enable",
-    "ivit_profile_read", "ivit_device_status", "ivit_last_launch_count", "ivit_destroy",
+    "ivit_get_changed", "ivit_get_cache", "ivit_reset", "ivit_timeline",
+    "ivit_timeline_read", "ivit_device_status", "ivit_last_launch_count", "ivit_destroy",
     "ivit_last_error", "ivit_select_noalloc", "ivit_action_combine",
 ]
 IVIT_NOALLOC_MAX_TOKENS = 65536
@@ -72,8 +72,9 @@ def load(path: str = LIB_PATH) -> C.CDLL:
     L.ivit_get_changed.argtypes = [P, I, P, P, P]
     L.ivit_get_cache.argtypes = [P, I, I, P, P]
     L.ivit_reset.argtypes = [P, I]
-    L.ivit_profile_enable.argtypes = [P, I]
-    L.ivit_profile_read.argtypes = [P, C.POINTER(C.c_double), C.POINTER(I64), C.POINTER(C.c_double)]
+    L.ivit_timeline.argtypes = [P, I]
+    L.ivit_timeline_read.argtypes = [P, P, C.POINTER(C.c_double), C.POINTER(I64), C.POINTER(C.c_double),
+                                     C.POINTER(C.c_double)]
     L.ivit_device_status.argtypes = [P, P]
     L.ivit_last_launch_count.restype = I64
     L.ivit_last_launch_count.argtypes = [P]
@@ -198,14 +199,24 @@ def ivit_reset(h: int, stream_index: int = -1) -> None:
     _check(load().ivit_reset(h, stream_index), h)
 
 
-def ivit_profile_enable(h: int, enable: bool) -> None:
-    _check(load().ivit_profile_enable(h, int(bool(enable))), h)
+def ivit_timeline(h: int, enable: bool) -> None:
+    """Timeline mode on or off (the encoder's CUDA graphs are captured again)."""
+    _check(load().ivit_timeline(h, int(bool(enable))), h)
 
 
-def ivit_profile_read(h: int) -> Tuple[float, int, float]:
-    ms, n, b = C.c_double(), C.c_int64(), C.c_double()
-    _check(load().ivit_profile_read(h, C.byref(ms), C.byref(n), C.byref(b)), h)
-    return ms.value, n.value, b.value
+TIMELINE_FAMILIES = ("gemm", "attention", "layernorm", "other")
+
+
+def ivit_timeline_read(h: int, stream=None) -> dict:
+    """Per-family kernel time (ms) and launches of the last call, the GEMM launches'
+    algorithmic bytes and the call's kernel span (ms); synchronises the stream."""
+    ms = (C.c_double * 4)()
+    n = (C.c_int64 * 4)()
+    b = C.c_double()
+    span = C.c_double()
+    _check(load().ivit_timeline_read(h, _stream(stream), ms, n, C.byref(b), C.byref(span)), h)
+    return {"ms": dict(zip(TIMELINE_FAMILIES, list(ms))), "launches": dict(zip(TIMELINE_FAMILIES, list(n))),
+            "gemm_bytes": b.value, "span_ms": span.value}
 
 
 def ivit_device_status(h: int, stream=None) -> int:

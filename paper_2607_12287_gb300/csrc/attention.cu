@@ -189,6 +189,7 @@ __global__ void __launch_bounds__(128, 1)
   }
   pdl_wait();  // queries and this call's K/V rows (QKV kernel) are visible from here
   pdl_launch_dependents();
+  stamp_begin(a.stamp);
 
   uint32_t ph_q = 0, ph_g = 0;  // completed phases: bq once per item, the others once per group
   bool ok = true;
@@ -434,6 +435,7 @@ __global__ void __launch_bounds__(128, 1)
   __syncthreads();
   tc_fence_after();
   if (warp == 0) tmem_dealloc(tmem, static_cast<uint32_t>(L.tm_cols));
+  stamp_end(a.stamp);
 }
 
 template <int DHP>

@@ -30,8 +30,13 @@ struct LayerW {
   CUtensorMap tm_ak, tm_av;  // the same caches, 64 x 128 boxes, 128-byte swizzle (tcgen05)
 };
 
-struct EventPair {
-  cudaEvent_t a, b;
+// Kernel families of the timeline.
+enum Family : int { kFamGemm = 0, kFamAttn = 1, kFamLN = 2, kFamOther = 3, kFamilies = 4 };
+
+struct TimelineSlot {
+  int family = kFamOther;
+  int n_out = 0, k = 0, kind = 0;  // GEMM shape and epilogue
+  int m_static = -1;               // GEMM rows when fixed, -1 when read from the device
 };
 
 // Launch shape of one GEMM: row-tile variant, CTAs per cluster (the K split), clusters.
@@ -163,11 +168,13 @@ struct ivit_handle {
   uint8_t* frames_buf = nullptr;
   int* counts_buf = nullptr;
 
-  bool profiling = false;
-  std::vector<EventPair> prof_events;
-  size_t prof_used = 0;
-  double prof_bytes = 0.0;
-  std::vector<double> call_static_bytes;  // per GEMM of the current call: weight bytes etc.
+  // Timeline mode (ivit_timeline): every launch of a call writes per-CTA start/end
+  // stamps into its slot of `stamps`; `slots_*` record each slot's kernel family and,
+  // for GEMMs, the shape that gives its algorithmic bytes.
+  bool timeline = false;
+  unsigned long long* stamps = nullptr;
+  int stamp_cap = 0, stamp_used = 0;
+  std::vector<TimelineSlot> slots_cur, slots_full, slots_inc, slots_last;
 
   std::string error;
 
@@ -699,12 +706,9 @@ void release(ivit_handle* h) {
   h->cap_stream = nullptr;
   if (h->wmem) cudaFree(h->wmem);
   if (h->smem) cudaFree(h->smem);
-  for (auto& e : h->prof_events) {
-    cudaEventDestroy(e.a);
-    cudaEventDestroy(e.b);
-  }
+  if (h->stamps) cudaFree(h->stamps);
+  h->stamps = nullptr;
   h->wmem = h->smem = nullptr;
-  h->prof_events.clear();
 }
 
 // Algorithmic bytes of one GEMM launch at M rows (weights, input rows, output rows, bias).
@@ -713,30 +717,29 @@ double gemm_bytes(int n_out, int k, int kind, long long M) {
   return 2.0 * n_out * k + 2.0 * M * k + out_b * M * n_out + 4.0 * n_out;
 }
 
+// Before each launch: the stamp slot of the launch in timeline mode (else none).
+void next_launch(ivit_handle* h, int family, const ivit::GemmArgs* ga = nullptr) {
+  ivit::g_stamp = nullptr;
+  if (!h->timeline || !h->stamps || h->stamp_used >= h->stamp_cap) return;
+  ivit::g_stamp = h->stamps + static_cast<size_t>(h->stamp_used++) * 2 * ivit::kStampCtas;
+  TimelineSlot sl;
+  sl.family = family;
+  if (ga) {
+    sl.n_out = ga->n_out;
+    sl.k = ga->k;
+    sl.kind = ga->epi.kind;
+    sl.m_static = ga->d_rows ? -1 : ga->m_static;
+  }
+  h->slots_cur.push_back(sl);
+}
+
 int gemm(ivit_handle* h, const GemmPlan& plan, const CUtensorMap& tw, const CUtensorMap& tx,
          ivit::GemmArgs a, cudaStream_t s) {
   a.err = h->err;
   a.partials = h->gemm_partials;
-  EventPair* ev = nullptr;
-  if (h->profiling) {
-    if (h->prof_used == h->prof_events.size()) {
-      EventPair e{};
-      IVIT_CK(h, cudaEventCreate(&e.a));
-      IVIT_CK(h, cudaEventCreate(&e.b));
-      h->prof_events.push_back(e);
-    }
-    ev = &h->prof_events[h->prof_used++];
-    IVIT_CK(h, cudaEventRecord(ev->a, s));
-  }
+  next_launch(h, kFamGemm, &a);
   IVIT_CK(h, ivit::launch_gemm(plan.bn, tw, tx, a, plan.n_clusters, plan.csize, s));
   ++h->launches;
-  if (ev) {
-    IVIT_CK(h, cudaEventRecord(ev->b, s));
-    h->call_static_bytes.push_back(a.n_out);  // n_out, k, kind, static M (or -1)
-    h->call_static_bytes.push_back(a.k);
-    h->call_static_bytes.push_back(a.epi.kind);
-    h->call_static_bytes.push_back(a.d_rows ? -1.0 : static_cast<double>(a.m_static));
-  }
   return IVIT_OK;
 }
 
@@ -838,8 +841,11 @@ int attention(ivit_handle* h, const LayerW& w, const bf16* ck, const bf16* cv, b
     at.qtiles = (N + 127) / 128;
     at.prefetch = full ? 0 : 1;
     at.key_splits = full ? h->attn_splits_full : h->attn_splits_inc;
+    next_launch(h, kFamAttn);
+    at.stamp = ivit::g_stamp;
     IVIT_CK(h, ivit::launch_attention_tc(h->tm_qa, w.tm_ak, w.tm_av, at, h->num_sms, s));
   } else {
+    next_launch(h, kFamAttn);
     IVIT_CK(h, ivit::launch_attention(w.tm_ck, w.tm_cv, h->q, ck, cv, h->cu_rows, h->rowtok, h->o, SV, N, D, h->H,
                                       full ? (N + 31) / 32 : std::max(1, (N / 10 + 31) / 32), s));
   }
@@ -862,6 +868,7 @@ int run_layers_mlp_all(ivit_handle* h, const GemmPlan* plan, bool full, cudaStre
     bf16* ck = h->cacheK + static_cast<size_t>(l) * M * D;
     bf16* cv = h->cacheV + static_cast<size_t>(l) * M * D;
     float* al = h->acache + static_cast<size_t>(l) * M * D;
+    next_launch(h, kFamLN);
     IVIT_CK(h, ivit::launch_layernorm_ex(total, h->x, nullptr, h->rowtok, w.ln1g, w.ln1b, h->xn, nullptr, D,
                                          c.ln_eps, M, h->row_grid, s));
     ++h->launches;
@@ -893,6 +900,7 @@ int run_layers_mlp_all(ivit_handle* h, const GemmPlan* plan, bool full, cudaStre
       a.epi.rowtok = h->rowtok;
       if (int r = gemm(h, plan[kGemmO], w.tm_o, h->tm_o, a, s)) return r;
     }
+    next_launch(h, kFamLN);
     IVIT_CK(h, ivit::launch_layernorm_ex(h->m_all, h->x, al, nullptr, w.ln2g, w.ln2b, h->xn, nullptr, D, c.ln_eps,
                                          M, h->row_grid, s));
     ++h->launches;
@@ -920,6 +928,7 @@ int run_layers_mlp_all(ivit_handle* h, const GemmPlan* plan, bool full, cudaStre
       if (int r = gemm(h, h->plan_full[kGemmDown], w.tm_2, h->tm_h, a, s)) return r;
     }
   }
+  next_launch(h, kFamLN);
   IVIT_CK(h, ivit::launch_layernorm(h->m_all, h->x, h->lnfg, h->lnfb, h->tok_out, nullptr, D, c.ln_eps, M,
                                     h->row_grid, s));
   ++h->launches;
@@ -938,8 +947,13 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
   const GemmPlan* plan = full ? h->plan_full : h->plan_inc;
   const int* total = h->cu_rows + SV;
   h->launches = 0;
-  h->call_static_bytes.clear();
+  h->slots_cur.clear();
+  h->stamp_used = 0;
+  if (h->timeline && h->stamps)  // CTAs that leave early write nothing: clear the last call's stamps
+    IVIT_CK(h, cudaMemsetAsync(h->stamps, 0, static_cast<size_t>(h->stamp_cap) * 2 * ivit::kStampCtas *
+                                                 sizeof(unsigned long long), s));
 
+  next_launch(h, kFamOther);
   IVIT_CK(h, ivit::launch_patchify(frames, h->patches, SV, c.img_h, c.img_w, c.patch, h->KPAD, s));
   ++h->launches;
   {
@@ -957,8 +971,10 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
   if (c.score_source == IVIT_SCORE_KEY0) {
     // Eq. 3 on first-layer keys of every token: W_K LN1(e + pos) + b_K (x, xn are free
     // until the updated rows are gathered below)
+    next_launch(h, kFamOther);
     IVIT_CK(h, ivit::launch_gather(h->m_all, h->rowtok_all, h->e_t, h->pos, h->x, nullptr, h->e_ref, N, D, 0,
                                    cm, M, h->row_grid, s));
+    next_launch(h, kFamLN);
     IVIT_CK(h, ivit::launch_layernorm(h->m_all, h->x, h->layers[0].ln1g, h->layers[0].ln1b, h->xn, nullptr, D,
                                       c.ln_eps, M, h->row_grid, s));
     h->launches += 2;
@@ -975,9 +991,11 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
     score_vec = h->key_t;
   }
   if (!full) {
+    next_launch(h, kFamOther);
     IVIT_CK(h, ivit::launch_score(score_vec, h->e_ref, h->sims, M, D, c.ref_mode == IVIT_REF_PREV_FRAME, s));
     ++h->launches;
   }
+  next_launch(h, kFamOther);
   IVIT_CK(h, ivit::launch_select(h->sims, N, SV, full ? IVIT_SEL_THRESHOLD : c.select_mode, c.threshold,
                                  c.topk, cm, h->idx, h->counts, h->cu_rows, h->rowtok, h->done_ctr,
                                  user_counts, s));
@@ -985,13 +1003,16 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
   if (c.mlp_tokens == IVIT_MLP_ALL) {
     // every token's residual stream (token-indexed), then the references of the updated
     // tokens (last-refresh mode, cold views) without touching x
+    next_launch(h, kFamOther);
     IVIT_CK(h, ivit::launch_gather(h->m_all, h->rowtok_all, h->e_t, h->pos, h->x, nullptr, h->e_ref, N, D, 0,
                                    cm, M, h->row_grid, s));
+    next_launch(h, kFamOther);
     IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, nullptr, score_vec, h->e_ref, N, D,
                                    c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
     h->launches += 2;
     return run_layers_mlp_all(h, plan, full, s);
   }
+  next_launch(h, kFamOther);
   IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, h->x, score_vec, h->e_ref, N, D,
                                  c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
   ++h->launches;
@@ -1013,7 +1034,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
     IVIT_CK(h, cudaMemsetAsync(h->pt_args.gbar, 0, 4 * sizeof(unsigned), s));
     IVIT_CK(h, ivit::launch_persistent(h->pt_args, h->pt_grid, h->pt_smem, s));
     ++h->launches;
-    if (h->pt_args.trace && !h->profiling) {
+    if (h->pt_args.trace && !h->timeline) {
       cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
       cudaStreamIsCapturing(s, &cs);
       if (cs == cudaStreamCaptureStatusNone) print_trace(h, s);
@@ -1024,6 +1045,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
     const LayerW& w = h->layers[l];
     bf16* ck = h->cacheK + static_cast<size_t>(l) * M * D;
     bf16* cv = h->cacheV + static_cast<size_t>(l) * M * D;
+    next_launch(h, kFamLN);
     IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln1g, w.ln1b, h->xn, nullptr, D, c.ln_eps, M,
                                       h->row_grid, s));
     ++h->launches;
@@ -1054,6 +1076,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
       a.epi.ld_out = D;
       if (int r = gemm(h, plan[kGemmO], w.tm_o, h->tm_o, a, s)) return r;
     }
+    next_launch(h, kFamLN);
     IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln2g, w.ln2b, h->xn, nullptr, D, c.ln_eps, M,
                                       h->row_grid, s));
     ++h->launches;
@@ -1081,6 +1104,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
       if (int r = gemm(h, plan[kGemmDown], w.tm_2, h->tm_h, a, s)) return r;
     }
   }
+  next_launch(h, kFamLN);
   IVIT_CK(h, ivit::launch_layernorm(total, h->x, h->lnfg, h->lnfb, h->tok_out, h->rowtok, D, c.ln_eps,
                                     M, h->row_grid, s));
   ++h->launches;
@@ -1101,6 +1125,7 @@ int capture(ivit_handle* h, bool full, cudaGraphExec_t* exec, int64_t* launches)
   cudaGraphDestroy(g);
   if (ei != cudaSuccess) return h->cuda_fail("cudaGraphInstantiate", ei);
   *launches = h->launches;
+  (full ? h->slots_full : h->slots_inc) = h->slots_cur;
   return IVIT_OK;
 }
 
@@ -1110,11 +1135,15 @@ int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_coun
   const size_t tok_bytes = static_cast<size_t>(h->M_max) * h->D * 2;
   bool any_cold = false;
   for (int v = 0; v < SV; ++v) any_cold = any_cold || h->cold[v];
-  if (h->use_graphs && !h->profiling && (full || !any_cold)) {
+  if (h->use_graphs && (full || !any_cold)) {
     cudaGraphExec_t* exec = full ? &h->graph_full : &h->graph_inc;
     int64_t* nl = full ? &h->graph_full_launches : &h->graph_inc_launches;
-    if (!*exec)
-      if (int r = capture(h, full, exec, nl)) return r;
+    if (!*exec) {
+      const int r = capture(h, full, exec, nl);
+      ivit::g_stamp = nullptr;
+      if (r) return r;
+    }
+    h->slots_last = full ? h->slots_full : h->slots_inc;
     const size_t fbytes = static_cast<size_t>(SV) * h->cfg.img_h * h->cfg.img_w * 3;
     IVIT_CK(h, cudaMemcpyAsync(h->frames_buf, frames, fbytes, cudaMemcpyDeviceToDevice, s));
     IVIT_CK(h, cudaGraphLaunch(*exec, s));
@@ -1123,22 +1152,14 @@ int run(ivit_handle* h, const uint8_t* frames, uint16_t* out, int32_t* user_coun
       IVIT_CK(h, cudaMemcpyAsync(user_counts, h->counts_buf, SV * sizeof(int), cudaMemcpyDeviceToDevice, s));
     h->launches = *nl;
   } else {
-    if (int r = run_core(h, frames, user_counts, full, s)) return r;
+    const int r = run_core(h, frames, user_counts, full, s);
+    ivit::g_stamp = nullptr;
+    if (r) return r;
+    h->slots_last = h->slots_cur;
     if (out) IVIT_CK(h, cudaMemcpyAsync(out, h->tok_out, tok_bytes, cudaMemcpyDeviceToDevice, s));
   }
   for (int v = 0; v < SV; ++v) h->cold[v] = 0;
 
-  if (h->profiling) {
-    int rows = 0;
-    IVIT_CK(h, cudaMemcpyAsync(&rows, h->cu_rows + SV, sizeof(int), cudaMemcpyDeviceToHost, s));
-    IVIT_CK(h, cudaStreamSynchronize(s));
-    for (size_t i = 0; i + 3 < h->call_static_bytes.size(); i += 4) {
-      const double m = h->call_static_bytes[i + 3] >= 0 ? h->call_static_bytes[i + 3] : rows;
-      h->prof_bytes += gemm_bytes(static_cast<int>(h->call_static_bytes[i]),
-                                  static_cast<int>(h->call_static_bytes[i + 1]),
-                                  static_cast<int>(h->call_static_bytes[i + 2]), static_cast<long long>(m));
-    }
-  }
   return IVIT_OK;
 }
 
@@ -1243,29 +1264,64 @@ int ivit_reset(ivit_handle* h, int stream_index) {
   return IVIT_OK;
 }
 
-int ivit_profile_enable(ivit_handle* h, int enable) {
+int ivit_timeline(ivit_handle* h, int enable) {
   if (!h) return IVIT_ERR_ARG;
-  h->profiling = enable != 0;
-  h->prof_used = 0;
-  h->prof_bytes = 0.0;
+  const bool on = enable != 0;
+  if (on && !h->stamps) {
+    h->stamp_cap = 512;
+    IVIT_CK(h, cudaMalloc(&h->stamps, static_cast<size_t>(h->stamp_cap) * 2 * ivit::kStampCtas *
+                                          sizeof(unsigned long long)));
+    IVIT_CK(h, cudaMemset(h->stamps, 0, static_cast<size_t>(h->stamp_cap) * 2 * ivit::kStampCtas *
+                                            sizeof(unsigned long long)));
+  }
+  if (on != h->timeline) {
+    // the graphs are captured again, with or without the stamps
+    IVIT_CK(h, cudaDeviceSynchronize());
+    if (h->graph_full) cudaGraphExecDestroy(h->graph_full);
+    if (h->graph_inc) cudaGraphExecDestroy(h->graph_inc);
+    h->graph_full = h->graph_inc = nullptr;
+    h->timeline = on;
+  }
   return IVIT_OK;
 }
 
-int ivit_profile_read(ivit_handle* h, double* gemm_ms_total, int64_t* gemm_launches,
-                      double* gemm_bytes_total) {
+int ivit_timeline_read(ivit_handle* h, void* stream, double* family_ms, int64_t* family_launches,
+                       double* gemm_bytes_total, double* span_ms) {
   if (!h) return IVIT_ERR_ARG;
-  double ms = 0.0;
-  for (size_t i = 0; i < h->prof_used; ++i) {
-    IVIT_CK(h, cudaEventSynchronize(h->prof_events[i].b));
-    float t = 0.f;
-    IVIT_CK(h, cudaEventElapsedTime(&t, h->prof_events[i].a, h->prof_events[i].b));
-    ms += t;
+  if (!h->timeline || !h->stamps) return h->fail(IVIT_ERR_ARG, "timeline mode is off");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t n = h->slots_last.size();
+  std::vector<unsigned long long> t(n * 2 * ivit::kStampCtas);
+  int rows = 0;
+  IVIT_CK(h, cudaMemcpyAsync(&rows, h->cu_rows + h->SV, sizeof(int), cudaMemcpyDeviceToHost, s));
+  if (n) IVIT_CK(h, cudaMemcpyAsync(t.data(), h->stamps, t.size() * sizeof(unsigned long long),
+                                    cudaMemcpyDeviceToHost, s));
+  IVIT_CK(h, cudaStreamSynchronize(s));
+  double ms[kFamilies] = {0}, bytes = 0;
+  int64_t cnt[kFamilies] = {0};
+  unsigned long long first = ~0ull, last = 0;
+  for (size_t i = 0; i < n; ++i) {
+    unsigned long long b = ~0ull, e = 0;
+    for (int c = 0; c < ivit::kStampCtas; ++c) {
+      const unsigned long long sb = t[(i * ivit::kStampCtas + c) * 2], se = t[(i * ivit::kStampCtas + c) * 2 + 1];
+      if (sb) b = std::min(b, sb);
+      if (se) e = std::max(e, se);
+    }
+    const TimelineSlot& sl = h->slots_last[i];
+    ++cnt[sl.family];
+    if (e > b && b != ~0ull) {
+      ms[sl.family] += 1e-6 * static_cast<double>(e - b);
+      first = std::min(first, b);
+      last = std::max(last, e);
+    }
+    if (sl.family == kFamGemm) bytes += gemm_bytes(sl.n_out, sl.k, sl.kind, sl.m_static >= 0 ? sl.m_static : rows);
   }
-  if (gemm_ms_total) *gemm_ms_total = ms;
-  if (gemm_launches) *gemm_launches = static_cast<int64_t>(h->prof_used);
-  if (gemm_bytes_total) *gemm_bytes_total = h->prof_bytes;
-  h->prof_used = 0;
-  h->prof_bytes = 0.0;
+  for (int f = 0; f < kFamilies; ++f) {
+    if (family_ms) family_ms[f] = ms[f];
+    if (family_launches) family_launches[f] = cnt[f];
+  }
+  if (gemm_bytes_total) *gemm_bytes_total = bytes;
+  if (span_ms) *span_ms = last > first ? 1e-6 * static_cast<double>(last - first) : 0.0;
   return IVIT_OK;
 }
 

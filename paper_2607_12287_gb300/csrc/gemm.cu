@@ -155,6 +155,7 @@ __global__ void __launch_bounds__(128, 1)
   }
   pdl_wait();  // outputs of the previous kernel on the stream are visible from here
   pdl_launch_dependents();
+  stamp_begin(a.stamp);
 
   uint32_t p_stage = 0, p_phase = 0;  // producer ring position
   uint32_t c_stage = 0, c_phase = 0;  // MMA ring position
@@ -302,6 +303,7 @@ __global__ void __launch_bounds__(128, 1)
     tc_fence_after();
     tmem_dealloc(tmem, BN_MAX);
   }
+  stamp_end(a.stamp);
 }
 
 // Many-tile form for single-CTA clusters (large row counts): a persistent loop over the
@@ -373,6 +375,7 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
   }
   pdl_wait();
   pdl_launch_dependents();
+  stamp_begin(a.stamp);
 
   if (warp == WS_EPI_WARPS) {
     if (lane == 0) {
@@ -483,6 +486,7 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
     tc_fence_after();
     tmem_dealloc(tmem, 2 * BN_MAX);
   }
+  stamp_end(a.stamp);
 }
 
 template <int BN>
@@ -555,7 +559,9 @@ int gemm_max_clusters(int bn_max, int csize) {
 }
 
 cudaError_t launch_gemm(int bn_max, const CUtensorMap& tm_w, const CUtensorMap& tm_x,
-                        const GemmArgs& a, int n_clusters, int csize, cudaStream_t s) {
+                        const GemmArgs& args, int n_clusters, int csize, cudaStream_t s) {
+  GemmArgs a = args;
+  a.stamp = g_stamp;
   if (bn_max == 64) return launch_variant<64>(tm_w, tm_x, a, n_clusters, csize, s);
   return launch_variant<256>(tm_w, tm_x, a, n_clusters, csize, s);
 }

@@ -14,6 +14,10 @@ using bf16 = __nv_bfloat16;
 // IVIT_NO_PDL environment variable turns it off at handle creation).
 extern bool g_use_pdl;
 
+// Stamp block (timeline mode) the next launch of this host thread passes to its kernel:
+// [kStampCtas][2] global times, or null.  Set by the engine before each launch.
+extern thread_local unsigned long long* g_stamp;
+
 // cudaLaunchKernelEx with optional cluster width and the PDL attribute.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
@@ -78,6 +82,7 @@ struct GemmArgs {
   // floats for every CTA of the launch.  Required when the launch's clusters have more
   // than one CTA.
   float* partials = nullptr;
+  unsigned long long* stamp = nullptr;  // timeline stamps of this launch (or null)
   GemmEpilogue epi;
 };
 
@@ -232,6 +237,7 @@ struct AttnTcArgs {
   int key_splits = 1;             // CTAs per cluster splitting the keys (1..8, N/splits <= 256)
   int prefetch = 0;               // 1: cached K/V loaded before the wait, then the updated
                                   //    rows re-read (incremental calls)
+  unsigned long long* stamp = nullptr;  // timeline stamps of this launch (or null)
 };
 
 // One-time function attributes of the tensor-core attention kernel.

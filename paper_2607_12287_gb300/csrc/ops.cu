@@ -7,6 +7,7 @@
 namespace ivit {
 
 bool g_use_pdl = true;
+thread_local unsigned long long* g_stamp = nullptr;
 
 namespace {
 
@@ -33,9 +34,10 @@ __device__ __forceinline__ bool is_cold(const ColdMask& m, int v) {
 // consecutive threads read and write contiguous runs; otherwise one thread per (token,
 // ky) row with byte loads.  Columns P*P*3 .. kpad-1 stay zero (set once at allocation).
 __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __restrict__ patches,
-                                int sv, int img_h, int img_w, int P, int kpad) {
+                                int sv, int img_h, int img_w, int P, int kpad, unsigned long long* stamp) {
   pdl_wait();
   pdl_launch_dependents();
+  stamp_begin(stamp);
   const int gw = img_w / P, gh = img_h / P, N = gw * gh;
   const int row = P * 3;
   const long long stride = static_cast<long long>(gridDim.x) * blockDim.x;
@@ -56,6 +58,7 @@ __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __rest
       *reinterpret_cast<__nv_bfloat162*>(patches + static_cast<size_t>(tok) * kpad + ky * row + 2 * j) =
           __floats2bfloat162_rn(static_cast<float>(b2 & 0xFF) - 128.f, static_cast<float>(b2 >> 8) - 128.f);
     }
+    stamp_end(stamp);
     return;
   }
   const long long total = static_cast<long long>(sv) * N * P;
@@ -69,6 +72,7 @@ __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __rest
     bf16* dst = patches + static_cast<size_t>(tok) * kpad + ky * row;
     for (int j = 0; j < row; ++j) dst[j] = __float2bfloat16_rn(static_cast<float>(src[j]) - 128.f);
   }
+  stamp_end(stamp);
 }
 
 // ------------------------------------------------------------------------ score
@@ -76,9 +80,11 @@ __global__ void patchify_kernel(const uint8_t* __restrict__ frames, bf16* __rest
 // per token, 128-bit loads.  With copy_ref the reference row is replaced by e_t
 // (reference = previous frame).
 __global__ void score_kernel(const float* __restrict__ e_t, float* __restrict__ e_ref,
-                             float* __restrict__ sims, int rows, int dim, int copy_ref) {
+                             float* __restrict__ sims, int rows, int dim, int copy_ref,
+                             unsigned long long* stamp) {
   pdl_wait();
   pdl_launch_dependents();
+  stamp_begin(stamp);
   const int warps = blockDim.x >> 5;
   const int lane = threadIdx.x & 31;
   for (int r = blockIdx.x * warps + (threadIdx.x >> 5); r < rows; r += gridDim.x * warps) {
@@ -97,6 +103,7 @@ __global__ void score_kernel(const float* __restrict__ e_t, float* __restrict__ 
     nb = warp_sum(nb);
     if (lane == 0) sims[r] = dot / fmaxf(sqrtf(na) * sqrtf(nb), 1e-12f);
   }
+  stamp_end(stamp);
 }
 
 // ----------------------------------------------------------------------- select
@@ -109,9 +116,10 @@ __global__ void select_kernel(const float* __restrict__ sims, int N, int sv, int
                               int topk, const ColdMask cold, int* __restrict__ idx,
                               int* __restrict__ counts, int* __restrict__ cu_rows,
                               int* __restrict__ rowtok, int* __restrict__ done_ctr,
-                              int* __restrict__ user_counts) {
+                              int* __restrict__ user_counts, unsigned long long* stamp) {
   pdl_wait();
   pdl_launch_dependents();
+  stamp_begin(stamp);
   extern __shared__ float s_sims[];  // [N]
   __shared__ int s_warp[32];
   __shared__ int s_last;
@@ -162,7 +170,10 @@ __global__ void select_kernel(const float* __restrict__ sims, int N, int sv, int
   __syncthreads();
   if (i == 0) s_last = (atomicAdd(done_ctr, 1) == sv - 1) ? 1 : 0;
   __syncthreads();
-  if (!s_last) return;
+  if (!s_last) {
+    stamp_end(stamp);
+    return;
+  }
   __threadfence();
   if (i == 0) {
     int acc = 0;
@@ -184,6 +195,7 @@ __global__ void select_kernel(const float* __restrict__ sims, int N, int sv, int
     const int k = r - __ldcg(cu_rows + lo);
     rowtok[r] = lo * N + __ldcg(idx + static_cast<size_t>(lo) * N + k);
   }
+  stamp_end(stamp);
 }
 
 // ----------------------------------------------------------------------- gather
@@ -195,9 +207,10 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
                               const float* __restrict__ e_t, const float* __restrict__ pos,
                               float* __restrict__ x, const float* __restrict__ ref_src,
                               float* __restrict__ e_ref, int N, int dim, int ref_last_refresh,
-                              const ColdMask cold) {
+                              const ColdMask cold, unsigned long long* stamp) {
   pdl_wait();
   pdl_launch_dependents();
+  stamp_begin(stamp);
   const int rows = *total_rows;
   const int warps = blockDim.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -220,6 +233,7 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
       for (int c = lane; c < dim / 4; c += 32) er[c] = src[c];
     }
   }
+  stamp_end(stamp);
 }
 
 // -------------------------------------------------------------------- layernorm
@@ -237,7 +251,7 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, float* __restric
                                  const float* __restrict__ add, const int* __restrict__ src_rowtok,
                                  const float* __restrict__ gamma, const float* __restrict__ beta,
                                  bf16* __restrict__ y, const int* __restrict__ dst_rowtok, int dim,
-                                 float eps) {
+                                 float eps, unsigned long long* stamp) {
   const int warps = blockDim.x >> 5;
   const int lane = threadIdx.x & 31;
   const int n4 = dim / 4;
@@ -254,6 +268,7 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, float* __restric
   const int rows = *nrows;
   pdl_wait();
   pdl_launch_dependents();
+  stamp_begin(stamp);
   for (int r = blockIdx.x * warps + (threadIdx.x >> 5); r < rows; r += gridDim.x * warps) {
     const size_t irow = kGather ? static_cast<size_t>(src_rowtok[r]) : static_cast<size_t>(r);
     const float4* xr = reinterpret_cast<const float4*>(static_cast<const float*>(x) + irow * dim);
@@ -292,6 +307,7 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, float* __restric
       }
     }
   }
+  stamp_end(stamp);
 }
 
 // -------------------------------------------------------------------- attention
@@ -520,13 +536,14 @@ cudaError_t launch_patchify(const uint8_t* frames, bf16* patches, int sv, int im
   if ((patch * 3) % 2 == 0) total *= patch * 3 / 2;
   const long long blocks = (total + 255) / 256;
   const int grid = static_cast<int>(blocks < 8192 ? blocks : 8192);
-  return launch_ex(patchify_kernel, dim3(grid), dim3(256), 0, s, 1, frames, patches, sv, img_h, img_w, patch, kpad);
+  return launch_ex(patchify_kernel, dim3(grid), dim3(256), 0, s, 1, frames, patches, sv, img_h, img_w, patch, kpad,
+                   g_stamp);
 }
 
 cudaError_t launch_score(const float* e_t, float* e_ref, float* sims, int rows, int dim,
                          int copy_ref, cudaStream_t s) {
   const int grid = min((rows + 7) / 8, 4096);
-  return launch_ex(score_kernel, dim3(grid), dim3(256), 0, s, 1, e_t, e_ref, sims, rows, dim, copy_ref);
+  return launch_ex(score_kernel, dim3(grid), dim3(256), 0, s, 1, e_t, e_ref, sims, rows, dim, copy_ref, g_stamp);
 }
 
 cudaError_t launch_select(const float* sims, int n_tok, int sv, int mode, float tau, int topk,
@@ -534,7 +551,7 @@ cudaError_t launch_select(const float* sims, int n_tok, int sv, int mode, float 
                           int* done_ctr, int* user_counts, cudaStream_t s) {
   const int threads = (n_tok + 31) / 32 * 32;
   return launch_ex(select_kernel, dim3(sv), dim3(threads), n_tok * sizeof(float), s, 1, sims, n_tok, sv,
-                   mode, tau, topk, cold, idx, counts, cu_rows, rowtok, done_ctr, user_counts);
+                   mode, tau, topk, cold, idx, counts, cu_rows, rowtok, done_ctr, user_counts, g_stamp);
 }
 
 cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const float* e_t,
@@ -543,7 +560,7 @@ cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const flo
                           cudaStream_t s) {
   grid = max(1, min(grid, (max_rows + 7) / 8));
   return launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, 1, cu_rows_total, rowtok, e_t, pos, x,
-                   ref_src, e_ref, n_tok, dim, ref_last_refresh, cold);
+                   ref_src, e_ref, n_tok, dim, ref_last_refresh, cold, g_stamp);
 }
 
 cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma, const float* beta,
@@ -560,7 +577,7 @@ cudaError_t launch_layernorm_ex(const int* rows, float* x, const float* add, con
   auto kern = add ? (src_rowtok ? layernorm_kernel<true, true> : layernorm_kernel<true, false>)
                   : (src_rowtok ? layernorm_kernel<false, true> : layernorm_kernel<false, false>);
   return launch_ex(kern, dim3(grid), dim3(256), 0, s, 1, rows, x, add, src_rowtok, gamma, beta, y, dst_rowtok, dim,
-                   eps);
+                   eps, g_stamp);
 }
 
 size_t attention_smem(int dh) {

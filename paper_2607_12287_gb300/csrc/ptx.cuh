@@ -308,6 +308,20 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
+// ------------------------------------------------------------- kernel timeline
+// Optional per-launch stamps (the library's timeline mode): thread 0 of CTA b writes
+// the global time after the kernel's wait on the previous kernel to s[2b] and the time
+// it finishes to s[2b+1]; only the first kStampCtas CTAs of a launch record.
+constexpr int kStampCtas = 1024;
+
+__device__ __forceinline__ void stamp_begin(unsigned long long* s) {
+  if (s && threadIdx.x == 0 && blockIdx.x < kStampCtas) s[2 * blockIdx.x] = globaltimer_ns();
+}
+
+__device__ __forceinline__ void stamp_end(unsigned long long* s) {
+  if (s && threadIdx.x == 0 && blockIdx.x < kStampCtas) s[2 * blockIdx.x + 1] = globaltimer_ns();
+}
+
 // ------------------------------------------------------ programmatic dependent launch
 // Every tcgen05 kernel allocates its TMEM columns before pdl_wait and calls
 // pdl_launch_dependents only after it.  So at most two grids overlap on an SM, every CTA

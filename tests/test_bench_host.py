@@ -5,6 +5,7 @@ import hashlib
 import os
 
 import bench
+from paper_2607_12287_gb300 import synth
 
 GEMM_SRC = os.path.join(bench.ROOT, "paper_2607_12287_gb300", "csrc", "gemm.cu")
 
@@ -64,3 +65,15 @@ def test_describe_names_the_workload():
     assert d["workload"] == "so400m_224_1view" and d["views"] == 1
     assert "dim 1152" in d["encoder"] and "27 layers" in d["encoder"]
     assert bench.describe(synth.sweep_workload(0.25))["selection"] == "top-64"
+
+
+def test_algorithmic_bytes_per_step_so400m():
+    # weights 823.5 MB of bf16 matrices + 27 layers of cached K/V (31.9 MB) + frame +
+    # embeddings + the updated rows' writes: about 0.86 GB for the 1-view 224 px stream
+    import bench
+    wl = synth.WORKLOADS["so400m_224_1view"]
+    w = bench.weight_matrix_bytes(wl.shape)
+    assert abs(w - 823.5e6) < 1.5e6
+    b = bench.algorithmic_bytes_per_step(wl, 26)
+    assert 0.85e9 < b < 0.87e9
+    assert bench.algorithmic_bytes_per_step(wl, 52) > b

@@ -276,3 +276,37 @@ def test_stream_kernel_row_passes(pkg, oracle_mod, forced_path, p):
     frames = list(synth.stream_random(shape, 2, 4, 152, change_p=p))
     stats = run_side_by_side(pkg, oracle_mod, shape, w, frames, 2, 1, check_caches=True)
     assert max(int(st[2].sum()) for st in stats[1:]) > 32
+
+
+def test_timeline_records_every_launch(pkg):
+    # timeline mode: the graph is captured again with per-launch stamps; the outputs are
+    # bitwise those of the plain graph, each family has its launches, and the kernels'
+    # times fit inside the call's span (each starts after the previous one completed)
+    import torch
+    shape = SHAPE_A
+    w = synth.make_weights(shape, 161)
+    frames = [torch.from_numpy(f).cuda() for f in synth.stream_random(shape, 3, 4, 162, change_p=0.2)]
+    outs = []
+    for tl in (False, True):
+        enc = pkg.IncrementalViT(shape, w, 1, 3)
+        try:
+            if tl:
+                pkg.ivit_timeline(enc.h, True)
+            enc.encode_full(frames[0])
+            got = [enc.encode_incremental(f)[0].clone() for f in frames[1:]]
+            outs.append(got)
+            if tl:
+                r = pkg.ivit_timeline_read(enc.h)
+                L = shape.depth
+                assert r["launches"] == {"gemm": 1 + 4 * L, "attention": L, "layernorm": 2 * L + 1, "other": 4}
+                assert all(v > 0 for v in r["ms"].values())
+                assert sum(r["ms"].values()) <= r["span_ms"] * 1.02
+                assert r["gemm_bytes"] > 2 * shape.dim * 3 * shape.dim * L
+                pkg.ivit_timeline(enc.h, False)
+                with pytest.raises(pkg.IvitError):
+                    pkg.ivit_timeline_read(enc.h)
+            assert enc.device_status() == 0
+        finally:
+            enc.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
