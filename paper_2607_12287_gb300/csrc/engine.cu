@@ -110,6 +110,17 @@ struct ivit_handle {
   int device = 0, num_sms = 0;
   int row_grid = 0;
   GemmPlan plan_full[kGemmSlots], plan_inc[kGemmSlots];
+  // Row-count bands of the incremental graph (band 0 = plan_inc): launch plans and
+  // attention key splits made for at most band_ub[b] updated rows; a switch node picks
+  // the band of each call's device-resident row count.
+  int n_bands = 1;
+  int band_ub[4] = {0, 0, 0, 0};
+  GemmPlan plan_band[4][kGemmSlots];
+  int attn_splits_band[4] = {1, 1, 1, 1};
+  bool capture_bands = false;  // set while the incremental graph is captured with bands
+  int known_band = -1;         // set while it is captured for a row count known in advance
+  ivit::RowBands bands;        // the switch node's handle and the bands' row bounds
+  cudaStream_t cap_stream2 = nullptr;  // captures the band bodies
 
   void* wmem = nullptr;  // weights (device)
   void* smem = nullptr;  // state + workspaces (device)
@@ -484,6 +495,19 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   IVIT_CK(h, ivit::attention_tc_setup());
   if (const char* at = std::getenv("IVIT_ATTN")) h->attn_tc = std::string(at) != "simt";
   {
+    // Row bands: the first holds a tenth of the tokens (rounded up to 16, at least 64),
+    // each next one twice the previous, the last all of them; at most four.
+    int ub = std::max(64, (static_cast<int>(M / 10) + 15) / 16 * 16);
+    h->n_bands = 0;
+    while (h->n_bands < 4) {
+      const bool last = ub >= static_cast<int>(M) || h->n_bands == 3;
+      h->band_ub[h->n_bands++] = last ? static_cast<int>(M) : ub;
+      if (last) break;
+      ub *= 2;
+    }
+    if (std::getenv("IVIT_NO_BANDS")) h->n_bands = 1;
+  }
+  {
     // Key splits of the tensor-core attention: as many as fill the SMs once for the
     // expected items (query tiles x heads x views: all tokens when full, a tenth when
     // incremental), at least 64 keys per CTA, one (online softmax over key groups) when
@@ -500,6 +524,8 @@ int setup(ivit_handle* h, const uint16_t* wb) {
     };
     h->attn_splits_full = splits(h->N);
     h->attn_splits_inc = splits(std::max(1, h->N / 10));
+    h->attn_splits_band[0] = h->attn_splits_inc;
+    for (int b = 1; b < h->n_bands; ++b) h->attn_splits_band[b] = splits(std::max(1, h->band_ub[b] / h->SV));
     if (ivit::attention_tc_smem(h->N, dh, h->attn_splits_full) > static_cast<size_t>(optin) ||
         ivit::attention_tc_smem(h->N, dh, h->attn_splits_inc) > static_cast<size_t>(optin))
       h->attn_tc = false;  // not reachable for N <= 1024, dh <= 128
@@ -507,6 +533,7 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   if (std::getenv("IVIT_NO_PDL")) ivit::g_use_pdl = false;
   if (std::getenv("IVIT_NO_GRAPH")) h->use_graphs = false;
   IVIT_CK(h, cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking));
+  IVIT_CK(h, cudaStreamCreateWithFlags(&h->cap_stream2, cudaStreamNonBlocking));
   h->row_grid = h->num_sms * 4;
   {
     // Full encodes know M = SV*N.  Incremental calls are planned for a tenth of the
@@ -520,6 +547,11 @@ int setup(ivit_handle* h, const uint16_t* wb) {
       h->plan_full[g] = plan_gemm(h->num_sms, bn_full, shapes[g][0], shapes[g][1], static_cast<int>(M));
       h->plan_inc[g] = g == kGemmEmbed ? h->plan_full[g]
                                        : plan_gemm(h->num_sms, bn_inc, shapes[g][0], shapes[g][1], m_inc);
+      h->plan_band[0][g] = h->plan_inc[g];
+      for (int b = 1; b < h->n_bands; ++b)
+        h->plan_band[b][g] = g == kGemmEmbed ? h->plan_full[g]
+                                             : plan_gemm(h->num_sms, h->band_ub[b] <= 64 ? 64 : 256, shapes[g][0],
+                                                         shapes[g][1], h->band_ub[b]);
     }
     if (std::getenv("IVIT_DEBUG")) {
       static const char* names[kGemmSlots] = {"embed", "qkv", "out", "up", "down"};
@@ -527,6 +559,8 @@ int setup(ivit_handle* h, const uint16_t* wb) {
         std::fprintf(stderr, "ivit gemm %-5s full bn=%d cluster=%d x %d | inc bn=%d cluster=%d x %d\n",
                      names[g], h->plan_full[g].bn, h->plan_full[g].csize, h->plan_full[g].n_clusters,
                      h->plan_inc[g].bn, h->plan_inc[g].csize, h->plan_inc[g].n_clusters);
+      for (int b = 1; b < h->n_bands; ++b)
+        std::fprintf(stderr, "ivit band %d (<= %d rows): attention splits %d\n", b, h->band_ub[b], h->attn_splits_band[b]);
     }
   }
 
@@ -626,8 +660,14 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   // slots for every plan: clusters x CTAs per cluster x row tile x 128 features, fp32
   size_t part_floats = 0;
   for (int g = 0; g < kGemmSlots; ++g)
+  {
     for (const GemmPlan* pl : {&h->plan_full[g], &h->plan_inc[g]})
       part_floats = std::max(part_floats, static_cast<size_t>(pl->n_clusters) * pl->csize * pl->bn * 128);
+    for (int b = 0; b < h->n_bands; ++b) {
+      const GemmPlan& pl = h->plan_band[b][g];
+      part_floats = std::max(part_floats, static_cast<size_t>(pl.n_clusters) * pl.csize * pl.bn * 128);
+    }
+  }
   const size_t o_gpart = sa.take(part_floats * 4);
   const size_t o_rta = sa.take(M * 4), o_mall = sa.take(4);
   const size_t o_fb = sa.take(static_cast<size_t>(h->SV) * c.img_h * c.img_w * 3);
@@ -702,6 +742,8 @@ void release(ivit_handle* h) {
   if (h->graph_full) cudaGraphExecDestroy(h->graph_full);
   if (h->graph_inc) cudaGraphExecDestroy(h->graph_inc);
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
+  if (h->cap_stream2) cudaStreamDestroy(h->cap_stream2);
+  h->cap_stream2 = nullptr;
   h->graph_full = h->graph_inc = nullptr;
   h->cap_stream = nullptr;
   if (h->wmem) cudaFree(h->wmem);
@@ -823,7 +865,8 @@ void print_stream_trace(ivit_handle* h, cudaStream_t s) {
 }
 
 // Attention of the updated queries over all tokens of their view for one layer.
-int attention(ivit_handle* h, const LayerW& w, const bf16* ck, const bf16* cv, bool full, cudaStream_t s) {
+int attention(ivit_handle* h, const LayerW& w, const bf16* ck, const bf16* cv, bool full, cudaStream_t s,
+              int key_splits = 0) {
   const int N = h->N, D = h->D, SV = h->SV;
   if (h->attn_tc) {
     ivit::AttnTcArgs at;
@@ -840,7 +883,7 @@ int attention(ivit_handle* h, const LayerW& w, const bf16* ck, const bf16* cv, b
     at.sv = SV;
     at.qtiles = (N + 127) / 128;
     at.prefetch = full ? 0 : 1;
-    at.key_splits = full ? h->attn_splits_full : h->attn_splits_inc;
+    at.key_splits = key_splits > 0 ? key_splits : (full ? h->attn_splits_full : h->attn_splits_inc);
     next_launch(h, kFamAttn);
     at.stamp = ivit::g_stamp;
     IVIT_CK(h, ivit::launch_attention_tc(h->tm_qa, w.tm_ak, w.tm_av, at, h->num_sms, s));
@@ -936,6 +979,116 @@ int run_layers_mlp_all(ivit_handle* h, const GemmPlan* plan, bool full, cudaStre
   return IVIT_OK;
 }
 
+// Per layer {LN1, QKV + K/V cache scatter (Eq. 4-5), attention, out-proj + residual,
+// LN2, MLP up + GELU, MLP down + residual}, then the final LN scattered into the
+// final-token cache, with the given launch plans and attention key splits.
+int run_layers(ivit_handle* h, const GemmPlan* plan, int attn_splits, bool full, cudaStream_t s) {
+  const ivit_config& c = h->cfg;
+  const int D = h->D, F = h->F, SV = h->SV, M = h->M_max;
+  const int* total = h->cu_rows + SV;
+  for (int l = 0; l < h->L; ++l) {
+    const LayerW& w = h->layers[l];
+    bf16* ck = h->cacheK + static_cast<size_t>(l) * M * D;
+    bf16* cv = h->cacheV + static_cast<size_t>(l) * M * D;
+    next_launch(h, kFamLN);
+    IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln1g, w.ln1b, h->xn, nullptr, D, c.ln_eps, M,
+                                      h->row_grid, s));
+    ++h->launches;
+    {
+      ivit::GemmArgs a;
+      a.n_out = 3 * D;
+      a.k = D;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiQKV;
+      a.epi.bias = w.bqkv;
+      a.epi.out_bf16 = h->q;
+      a.epi.ld_out = D;
+      a.epi.cache_k = ck;
+      a.epi.cache_v = cv;
+      a.epi.rowtok = h->rowtok;
+      a.epi.dim = D;
+      if (int r = gemm(h, plan[kGemmQKV], w.tm_qkv, h->tm_xn, a, s)) return r;
+    }
+    if (int r = attention(h, w, ck, cv, full, s, attn_splits)) return r;
+    {
+      ivit::GemmArgs a;
+      a.n_out = D;
+      a.k = D;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiResid;
+      a.epi.bias = w.bo;
+      a.epi.out_f32 = h->x;
+      a.epi.ld_out = D;
+      if (int r = gemm(h, plan[kGemmO], w.tm_o, h->tm_o, a, s)) return r;
+    }
+    next_launch(h, kFamLN);
+    IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln2g, w.ln2b, h->xn, nullptr, D, c.ln_eps, M,
+                                      h->row_grid, s));
+    ++h->launches;
+    {
+      ivit::GemmArgs a;
+      a.n_out = F;
+      a.k = D;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiGelu;
+      a.epi.bias = w.b1;
+      a.epi.out_bf16 = h->hbuf;
+      a.epi.ld_out = F;
+      a.epi.gelu_mode = c.gelu;
+      if (int r = gemm(h, plan[kGemmUp], w.tm_1, h->tm_xn, a, s)) return r;
+    }
+    {
+      ivit::GemmArgs a;
+      a.n_out = D;
+      a.k = F;
+      a.d_rows = total;
+      a.epi.kind = ivit::kEpiResid;
+      a.epi.bias = w.b2;
+      a.epi.out_f32 = h->x;
+      a.epi.ld_out = D;
+      if (int r = gemm(h, plan[kGemmDown], w.tm_2, h->tm_h, a, s)) return r;
+    }
+  }
+  next_launch(h, kFamLN);
+  IVIT_CK(h, ivit::launch_layernorm(total, h->x, h->lnfg, h->lnfb, h->tok_out, h->rowtok, D, c.ln_eps,
+                                    M, h->row_grid, s));
+  ++h->launches;
+  return IVIT_OK;
+}
+
+// Under capture of an incremental graph with row bands: a switch node after the
+// gather (which sets its value from the row count) with one body per band, each the
+// layer chain with that band's launch plans, captured on a second stream.  The
+// launches of one body count for the call.
+int capture_band_bodies(ivit_handle* h, cudaStream_t s) {
+  cudaStreamCaptureStatus st;
+  cudaGraph_t graph = nullptr;
+  const cudaGraphNode_t* deps = nullptr;
+  size_t ndeps = 0;
+  IVIT_CK(h, cudaStreamGetCaptureInfo(s, &st, nullptr, &graph, &deps, nullptr, &ndeps));
+  cudaGraphNodeParams np = {};
+  np.type = cudaGraphNodeTypeConditional;
+  np.conditional.handle = static_cast<cudaGraphConditionalHandle>(h->bands.handle);
+  np.conditional.type = cudaGraphCondTypeSwitch;
+  np.conditional.size = static_cast<unsigned>(h->n_bands);
+  cudaGraphNode_t node;
+  IVIT_CK(h, cudaGraphAddNode(&node, graph, deps, nullptr, ndeps, &np));
+  IVIT_CK(h, cudaStreamUpdateCaptureDependencies(s, &node, nullptr, 1, cudaStreamSetCaptureDependencies));
+  const int64_t pre = h->launches;
+  for (int b = 0; b < h->n_bands; ++b) {
+    h->launches = pre;
+    IVIT_CK(h, cudaStreamBeginCaptureToGraph(h->cap_stream2, np.conditional.phGraph_out[b], nullptr, nullptr, 0,
+                                             cudaStreamCaptureModeThreadLocal));
+    // (the band of every row attends like a full encode: no cached-K/V prefetch to patch)
+    const int r = run_layers(h, h->plan_band[b], h->attn_splits_band[b], h->band_ub[b] >= h->M_max, h->cap_stream2);
+    cudaGraph_t body = nullptr;
+    const cudaError_t e = cudaStreamEndCapture(h->cap_stream2, &body);
+    if (r) return r;
+    if (e != cudaSuccess) return h->cuda_fail("cudaStreamEndCapture (band body)", e);
+  }
+  return IVIT_OK;
+}
+
 // Enqueues the whole chain for one frame per view on `s` (eagerly or under capture).
 int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool full, cudaStream_t s) {
   const ivit_config& c = h->cfg;
@@ -1012,9 +1165,21 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
     h->launches += 2;
     return run_layers_mlp_all(h, plan, full, s);
   }
+  ivit::RowBands bands;  // (no switch node: handle 0)
+  if (h->capture_bands) {
+    cudaStreamCaptureStatus st;
+    cudaGraph_t graph = nullptr;
+    IVIT_CK(h, cudaStreamGetCaptureInfo(s, &st, nullptr, &graph));
+    cudaGraphConditionalHandle ch;
+    IVIT_CK(h, cudaGraphConditionalHandleCreate(&ch, graph, 0, cudaGraphCondAssignDefault));
+    bands.handle = static_cast<unsigned long long>(ch);
+    bands.n = h->n_bands;
+    for (int b = 0; b < h->n_bands; ++b) bands.ub[b] = h->band_ub[b];
+    h->bands = bands;
+  }
   next_launch(h, kFamOther);
   IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, h->x, score_vec, h->e_ref, N, D,
-                                 c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
+                                 c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s, bands));
   ++h->launches;
 
   bool any_cold = false;
@@ -1041,77 +1206,47 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
     }
     return IVIT_OK;
   }
-  for (int l = 0; l < h->L; ++l) {
-    const LayerW& w = h->layers[l];
-    bf16* ck = h->cacheK + static_cast<size_t>(l) * M * D;
-    bf16* cv = h->cacheV + static_cast<size_t>(l) * M * D;
-    next_launch(h, kFamLN);
-    IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln1g, w.ln1b, h->xn, nullptr, D, c.ln_eps, M,
-                                      h->row_grid, s));
-    ++h->launches;
-    {
-      ivit::GemmArgs a;
-      a.n_out = 3 * D;
-      a.k = D;
-      a.d_rows = total;
-      a.epi.kind = ivit::kEpiQKV;
-      a.epi.bias = w.bqkv;
-      a.epi.out_bf16 = h->q;
-      a.epi.ld_out = D;
-      a.epi.cache_k = ck;
-      a.epi.cache_v = cv;
-      a.epi.rowtok = h->rowtok;
-      a.epi.dim = D;
-      if (int r = gemm(h, plan[kGemmQKV], w.tm_qkv, h->tm_xn, a, s)) return r;
-    }
-    if (int r = attention(h, w, ck, cv, full, s)) return r;
-    {
-      ivit::GemmArgs a;
-      a.n_out = D;
-      a.k = D;
-      a.d_rows = total;
-      a.epi.kind = ivit::kEpiResid;
-      a.epi.bias = w.bo;
-      a.epi.out_f32 = h->x;
-      a.epi.ld_out = D;
-      if (int r = gemm(h, plan[kGemmO], w.tm_o, h->tm_o, a, s)) return r;
-    }
-    next_launch(h, kFamLN);
-    IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln2g, w.ln2b, h->xn, nullptr, D, c.ln_eps, M,
-                                      h->row_grid, s));
-    ++h->launches;
-    {
-      ivit::GemmArgs a;
-      a.n_out = F;
-      a.k = D;
-      a.d_rows = total;
-      a.epi.kind = ivit::kEpiGelu;
-      a.epi.bias = w.b1;
-      a.epi.out_bf16 = h->hbuf;
-      a.epi.ld_out = F;
-      a.epi.gelu_mode = c.gelu;
-      if (int r = gemm(h, plan[kGemmUp], w.tm_1, h->tm_xn, a, s)) return r;
-    }
-    {
-      ivit::GemmArgs a;
-      a.n_out = D;
-      a.k = F;
-      a.d_rows = total;
-      a.epi.kind = ivit::kEpiResid;
-      a.epi.bias = w.b2;
-      a.epi.out_f32 = h->x;
-      a.epi.ld_out = D;
-      if (int r = gemm(h, plan[kGemmDown], w.tm_2, h->tm_h, a, s)) return r;
-    }
-  }
-  next_launch(h, kFamLN);
-  IVIT_CK(h, ivit::launch_layernorm(total, h->x, h->lnfg, h->lnfb, h->tok_out, h->rowtok, D, c.ln_eps,
-                                    M, h->row_grid, s));
-  ++h->launches;
-  return IVIT_OK;
+  if (h->capture_bands) return capture_band_bodies(h, s);
+  if (!full && h->known_band >= 0)  // top-k: the row count is fixed, so is its band
+    return run_layers(h, h->plan_band[h->known_band], h->attn_splits_band[h->known_band],
+                      h->band_ub[h->known_band] >= h->M_max, s);
+  return run_layers(h, plan, full ? h->attn_splits_full : h->attn_splits_inc, full, s);
 }
 
+int capture_once(ivit_handle* h, bool full, cudaGraphExec_t* exec, int64_t* launches);
+
+// The incremental graph of the kernel chain is captured with a switch over the row
+// bands when there are several; if that capture fails the plain graph (band 0's plans
+// for every row count) is captured instead.
 int capture(ivit_handle* h, bool full, cudaGraphExec_t* exec, int64_t* launches) {
+  const bool chain = h->cfg.mlp_tokens == IVIT_MLP_UPDATED && !h->stream_ok && !h->persistent_inc;
+  if (!full && chain && h->n_bands > 1 && h->cfg.select_mode == IVIT_SEL_TOPK) {
+    // top-k (no cold view in a captured call): exactly k rows per view, so the band is
+    // known when the graph is captured and no switch is needed
+    const long long m = std::min<long long>(static_cast<long long>(h->cfg.topk), h->N) * h->SV;
+    int b = 0;
+    while (b + 1 < h->n_bands && m > h->band_ub[b]) ++b;
+    h->known_band = b;
+    const int r = capture_once(h, full, exec, launches);
+    h->known_band = -1;
+    return r;
+  }
+  // threshold selection: the row count is known only on the device; the switch pays its
+  // fixed cost (no programmatic overlap across the node) when a tenth of the tokens
+  // already exceeds 32 rows, so that row counts commonly cross bands
+  if (!full && chain && h->n_bands > 1 && h->M_max / 10 > 32) {
+    h->capture_bands = true;
+    const int r = capture_once(h, full, exec, launches);
+    h->capture_bands = false;
+    if (r == IVIT_OK) return IVIT_OK;
+    if (std::getenv("IVIT_DEBUG")) std::fprintf(stderr, "ivit: row-band graph failed (%s)\n", h->error.c_str());
+    cudaGetLastError();
+    h->n_bands = 1;
+  }
+  return capture_once(h, full, exec, launches);
+}
+
+int capture_once(ivit_handle* h, bool full, cudaGraphExec_t* exec, int64_t* launches) {
   IVIT_CK(h, cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal));
   const int r = run_core(h, h->frames_buf, h->counts_buf, full, h->cap_stream);
   cudaGraph_t g = nullptr;
@@ -1308,8 +1443,9 @@ int ivit_timeline_read(ivit_handle* h, void* stream, double* family_ms, int64_t*
       if (se) e = std::max(e, se);
     }
     const TimelineSlot& sl = h->slots_last[i];
+    if (b == ~0ull) continue;  // not run (another row band's body of the graph)
     ++cnt[sl.family];
-    if (e > b && b != ~0ull) {
+    if (e > b) {
       ms[sl.family] += 1e-6 * static_cast<double>(e - b);
       first = std::min(first, b);
       last = std::max(last, e);

@@ -189,12 +189,22 @@ cudaError_t launch_select(const float* sims, int n_tok, int sv, int mode, float 
                           const ColdMask& cold, int* idx, int* counts, int* cu_rows, int* rowtok,
                           int* done_ctr, int* user_counts, cudaStream_t s);
 
+// Row-count bands of an incremental call's CUDA graph: the launch plans of band b are
+// made for at most ub[b] updated rows; the graph's switch node runs the body of the
+// smallest band that holds the call's row count.
+struct RowBands {
+  unsigned long long handle = 0;  // cudaGraphConditionalHandle of the switch node (0: none)
+  int n = 0;
+  int ub[4] = {0, 0, 0, 0};
+};
+
 // x[r] = e_t[tok] + pos[tok % N] for the packed rows; refreshes e_ref[tok] from
-// ref_src[tok] for refreshed tokens (last-refresh reference or cold view).
+// ref_src[tok] for refreshed tokens (last-refresh reference or cold view).  With
+// bands.handle set, thread 0 of CTA 0 also selects the band of the row count.
 cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const float* e_t,
                           const float* pos, float* x, const float* ref_src, float* e_ref, int n_tok,
                           int dim, int ref_last_refresh, const ColdMask& cold, int max_rows, int grid,
-                          cudaStream_t s);
+                          cudaStream_t s, const RowBands& bands = RowBands());
 
 // y[r] = LN(x[r]) (bf16) for r < *rows; when dst_rowtok is set, row r is written to
 // row dst_rowtok[r] of y instead (final-token cache scatter).

@@ -207,11 +207,16 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
                               const float* __restrict__ e_t, const float* __restrict__ pos,
                               float* __restrict__ x, const float* __restrict__ ref_src,
                               float* __restrict__ e_ref, int N, int dim, int ref_last_refresh,
-                              const ColdMask cold, unsigned long long* stamp) {
+                              const ColdMask cold, const RowBands bands, unsigned long long* stamp) {
   pdl_wait();
   pdl_launch_dependents();
   stamp_begin(stamp);
   const int rows = *total_rows;
+  if (bands.handle && blockIdx.x == 0 && threadIdx.x == 0) {
+    unsigned b = 0;
+    while (b + 1 < static_cast<unsigned>(bands.n) && rows > bands.ub[b]) ++b;
+    cudaGraphSetConditional(static_cast<cudaGraphConditionalHandle>(bands.handle), b);
+  }
   const int warps = blockDim.x >> 5;
   const int lane = threadIdx.x & 31;
   for (int r = blockIdx.x * warps + (threadIdx.x >> 5); r < rows; r += gridDim.x * warps) {
@@ -557,10 +562,10 @@ cudaError_t launch_select(const float* sims, int n_tok, int sv, int mode, float 
 cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const float* e_t,
                           const float* pos, float* x, const float* ref_src, float* e_ref, int n_tok,
                           int dim, int ref_last_refresh, const ColdMask& cold, int max_rows, int grid,
-                          cudaStream_t s) {
+                          cudaStream_t s, const RowBands& bands) {
   grid = max(1, min(grid, (max_rows + 7) / 8));
   return launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, 1, cu_rows_total, rowtok, e_t, pos, x,
-                   ref_src, e_ref, n_tok, dim, ref_last_refresh, cold, g_stamp);
+                   ref_src, e_ref, n_tok, dim, ref_last_refresh, cold, bands, g_stamp);
 }
 
 cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma, const float* beta,
