@@ -1452,6 +1452,30 @@ int ivit_timeline_read(ivit_handle* h, void* stream, double* family_ms, int64_t*
     }
     if (sl.family == kFamGemm) bytes += gemm_bytes(sl.n_out, sl.k, sl.kind, sl.m_static >= 0 ? sl.m_static : rows);
   }
+  if (std::getenv("IVIT_DEBUG")) {  // mean launch time per family and GEMM epilogue kind
+    double kms[kFamilies][8] = {};
+    int kn[kFamilies][8] = {};
+    for (size_t i = 0; i < n; ++i) {
+      unsigned long long b = ~0ull, e = 0;
+      for (int c = 0; c < ivit::kStampCtas; ++c) {
+        const unsigned long long sb = t[(i * ivit::kStampCtas + c) * 2], se = t[(i * ivit::kStampCtas + c) * 2 + 1];
+        if (sb) b = std::min(b, sb);
+        if (se) e = std::max(e, se);
+      }
+      const TimelineSlot& sl = h->slots_last[i];
+      const int k = sl.family == kFamGemm ? std::min(7, std::max(0, sl.kind)) : 0;
+      if (e > b && b != ~0ull) {
+        kms[sl.family][k] += 1e-3 * static_cast<double>(e - b);
+        ++kn[sl.family][k];
+      }
+    }
+    static const char* fam[kFamilies] = {"gemm", "attention", "layernorm", "other"};
+    for (int f = 0; f < kFamilies; ++f)
+      for (int k = 0; k < 8; ++k)
+        if (kn[f][k])
+          std::fprintf(stderr, "ivit timeline: %s%s%d: %d launches, %.2f us each\n", fam[f], f == kFamGemm ? " epilogue " : " ",
+                       k, kn[f][k], kms[f][k] / kn[f][k]);
+  }
   for (int f = 0; f < kFamilies; ++f) {
     if (family_ms) family_ms[f] = ms[f];
     if (family_launches) family_launches[f] = cnt[f];
