@@ -760,12 +760,13 @@ double gemm_bytes(int n_out, int k, int kind, long long M) {
 }
 
 // Before each launch: the stamp slot of the launch in timeline mode (else none).
-void next_launch(ivit_handle* h, int family, const ivit::GemmArgs* ga = nullptr) {
+void next_launch(ivit_handle* h, int family, const ivit::GemmArgs* ga = nullptr, int other_kind = 0) {
   ivit::g_stamp = nullptr;
   if (!h->timeline || !h->stamps || h->stamp_used >= h->stamp_cap) return;
   ivit::g_stamp = h->stamps + static_cast<size_t>(h->stamp_used++) * 2 * ivit::kStampCtas;
   TimelineSlot sl;
   sl.family = family;
+  sl.kind = other_kind;
   if (ga) {
     sl.n_out = ga->n_out;
     sl.k = ga->k;
@@ -1106,7 +1107,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
     IVIT_CK(h, cudaMemsetAsync(h->stamps, 0, static_cast<size_t>(h->stamp_cap) * 2 * ivit::kStampCtas *
                                                  sizeof(unsigned long long), s));
 
-  next_launch(h, kFamOther);
+  next_launch(h, kFamOther, nullptr, 0);  // patchify
   IVIT_CK(h, ivit::launch_patchify(frames, h->patches, SV, c.img_h, c.img_w, c.patch, h->KPAD, s));
   ++h->launches;
   {
@@ -1124,7 +1125,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
   if (c.score_source == IVIT_SCORE_KEY0) {
     // Eq. 3 on first-layer keys of every token: W_K LN1(e + pos) + b_K (x, xn are free
     // until the updated rows are gathered below)
-    next_launch(h, kFamOther);
+    next_launch(h, kFamOther, nullptr, 3);  // gather
     IVIT_CK(h, ivit::launch_gather(h->m_all, h->rowtok_all, h->e_t, h->pos, h->x, nullptr, h->e_ref, N, D, 0,
                                    cm, M, h->row_grid, s));
     next_launch(h, kFamLN);
@@ -1144,11 +1145,11 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
     score_vec = h->key_t;
   }
   if (!full) {
-    next_launch(h, kFamOther);
+    next_launch(h, kFamOther, nullptr, 1);  // score
     IVIT_CK(h, ivit::launch_score(score_vec, h->e_ref, h->sims, M, D, c.ref_mode == IVIT_REF_PREV_FRAME, s));
     ++h->launches;
   }
-  next_launch(h, kFamOther);
+  next_launch(h, kFamOther, nullptr, 2);  // select
   IVIT_CK(h, ivit::launch_select(h->sims, N, SV, full ? IVIT_SEL_THRESHOLD : c.select_mode, c.threshold,
                                  c.topk, cm, h->idx, h->counts, h->cu_rows, h->rowtok, h->done_ctr,
                                  user_counts, s));
@@ -1156,10 +1157,10 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
   if (c.mlp_tokens == IVIT_MLP_ALL) {
     // every token's residual stream (token-indexed), then the references of the updated
     // tokens (last-refresh mode, cold views) without touching x
-    next_launch(h, kFamOther);
+    next_launch(h, kFamOther, nullptr, 3);  // gather
     IVIT_CK(h, ivit::launch_gather(h->m_all, h->rowtok_all, h->e_t, h->pos, h->x, nullptr, h->e_ref, N, D, 0,
                                    cm, M, h->row_grid, s));
-    next_launch(h, kFamOther);
+    next_launch(h, kFamOther, nullptr, 3);  // gather
     IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, nullptr, score_vec, h->e_ref, N, D,
                                    c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s));
     h->launches += 2;
@@ -1177,7 +1178,7 @@ int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool f
     for (int b = 0; b < h->n_bands; ++b) bands.ub[b] = h->band_ub[b];
     h->bands = bands;
   }
-  next_launch(h, kFamOther);
+  next_launch(h, kFamOther, nullptr, 3);  // gather
   IVIT_CK(h, ivit::launch_gather(total, h->rowtok, h->e_t, h->pos, h->x, score_vec, h->e_ref, N, D,
                                  c.ref_mode == IVIT_REF_LAST_REFRESH, cm, M, h->row_grid, s, bands));
   ++h->launches;
@@ -1463,7 +1464,7 @@ int ivit_timeline_read(ivit_handle* h, void* stream, double* family_ms, int64_t*
         if (se) e = std::max(e, se);
       }
       const TimelineSlot& sl = h->slots_last[i];
-      const int k = sl.family == kFamGemm ? std::min(7, std::max(0, sl.kind)) : 0;
+      const int k = std::min(7, std::max(0, sl.kind));
       if (e > b && b != ~0ull) {
         kms[sl.family][k] += 1e-3 * static_cast<double>(e - b);
         ++kn[sl.family][k];

@@ -1,6 +1,9 @@
 // Memory-bound kernels of the incremental encode: patchify, change score (Eq. 3),
 // selection + stream compaction, gather of the updated rows, layer norm (with the
 // final-token cache scatter), and attention of the updated queries over all tokens.
+#include <cstdlib>
+#include <cstring>
+
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -237,6 +240,70 @@ __global__ void gather_kernel(const int* __restrict__ total_rows, const int* __r
       float4* er = reinterpret_cast<float4*>(e_ref + static_cast<size_t>(tok) * dim);
       for (int c = lane; c < dim / 4; c += 32) er[c] = src[c];
     }
+  }
+  stamp_end(stamp);
+}
+
+// The same gather with the rows staged through shared memory by TMA bulk copies: per
+// group of GATHER_RPC rows one thread issues a cp.async.bulk of each row of e_t and of
+// the position embedding (contiguous, 16-byte aligned), every thread waits on the
+// group's mbarrier, then sums from shared memory into x with 128-bit stores.
+constexpr int GATHER_RPC = 4;
+
+__global__ void gather_bulk_kernel(const int* __restrict__ total_rows, const int* __restrict__ rowtok,
+                                   const float* __restrict__ e_t, const float* __restrict__ pos,
+                                   float* __restrict__ x, const float* __restrict__ ref_src,
+                                   float* __restrict__ e_ref, int N, int dim, int ref_last_refresh,
+                                   const ColdMask cold, const RowBands bands, unsigned long long* stamp) {
+  extern __shared__ __align__(128) float gsm[];  // [RPC][dim] e_t rows, then [RPC][dim] pos rows
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int s_tok[GATHER_RPC];
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(&bar), 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  pdl_wait();
+  pdl_launch_dependents();
+  stamp_begin(stamp);
+  const int rows = *total_rows;
+  if (bands.handle && blockIdx.x == 0 && threadIdx.x == 0) {
+    unsigned b = 0;
+    while (b + 1 < static_cast<unsigned>(bands.n) && rows > bands.ub[b]) ++b;
+    cudaGraphSetConditional(static_cast<cudaGraphConditionalHandle>(bands.handle), b);
+  }
+  const int n4 = dim / 4;
+  const uint32_t row_bytes = static_cast<uint32_t>(dim) * 4;
+  float4* se = reinterpret_cast<float4*>(gsm);
+  float4* sp = reinterpret_cast<float4*>(gsm + GATHER_RPC * dim);
+  uint32_t phase = 0;
+  for (int r0 = blockIdx.x * GATHER_RPC; r0 < rows; r0 += gridDim.x * GATHER_RPC, phase ^= 1u) {
+    const int nr = min(GATHER_RPC, rows - r0);
+    if (threadIdx.x == 0) {
+      mbar_arrive_expect_tx(smem_u32(&bar), 2u * nr * row_bytes);
+      for (int i = 0; i < nr; ++i) {
+        const int tok = rowtok[r0 + i];
+        s_tok[i] = tok;
+        bulk_load(smem_u32(se + i * n4), e_t + static_cast<size_t>(tok) * dim, row_bytes, smem_u32(&bar));
+        bulk_load(smem_u32(sp + i * n4), pos + static_cast<size_t>(tok % N) * dim, row_bytes, smem_u32(&bar));
+      }
+    }
+    // one vote both publishes s_tok and keeps the loop uniform when a wait gives up
+    if (__syncthreads_or(!mbar_wait(smem_u32(&bar), phase))) {
+      if (threadIdx.x == 0) mbar_wait(smem_u32(&bar), phase);  // the copies in flight (bounded)
+      break;
+    }
+    for (int e = threadIdx.x; e < nr * n4; e += blockDim.x) {
+      const int i = e / n4, c = e - i * n4;
+      const int tok = s_tok[i];
+      const float4 u = se[i * n4 + c], w = sp[i * n4 + c];
+      if (x) reinterpret_cast<float4*>(x + static_cast<size_t>(r0 + i) * dim)[c] =
+          make_float4(u.x + w.x, u.y + w.y, u.z + w.z, u.w + w.w);
+      if (ref_src && (ref_last_refresh || is_cold(cold, tok / N)))
+        reinterpret_cast<float4*>(e_ref + static_cast<size_t>(tok) * dim)[c] =
+            ref_src == e_t ? u : reinterpret_cast<const float4*>(ref_src + static_cast<size_t>(tok) * dim)[c];
+    }
+    __syncthreads();  // the tiles are read before the next group's copies overwrite them
   }
   stamp_end(stamp);
 }
@@ -563,6 +630,21 @@ cudaError_t launch_gather(const int* cu_rows_total, const int* rowtok, const flo
                           const float* pos, float* x, const float* ref_src, float* e_ref, int n_tok,
                           int dim, int ref_last_refresh, const ColdMask& cold, int max_rows, int grid,
                           cudaStream_t s, const RowBands& bands) {
+  const char* genv = std::getenv("IVIT_GATHER");  // read per launch: graphs capture it once
+  const bool bulk = genv && std::strcmp(genv, "tma") == 0;
+  if (bulk && dim % 4 == 0 && dim <= 2048) {
+    const size_t smem = 2 * GATHER_RPC * static_cast<size_t>(dim) * sizeof(float);
+    static bool attr = false;
+    if (!attr) {
+      const cudaError_t e = cudaFuncSetAttribute(gather_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 static_cast<int>(2 * GATHER_RPC * 2048 * sizeof(float)));
+      if (e != cudaSuccess) return e;
+      attr = true;
+    }
+    grid = max(1, min(grid, (max_rows + GATHER_RPC - 1) / GATHER_RPC));
+    return launch_ex(gather_bulk_kernel, dim3(grid), dim3(256), smem, s, 1, cu_rows_total, rowtok, e_t, pos, x,
+                     ref_src, e_ref, n_tok, dim, ref_last_refresh, cold, bands, g_stamp);
+  }
   grid = max(1, min(grid, (max_rows + 7) / 8));
   return launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, 1, cu_rows_total, rowtok, e_t, pos, x,
                    ref_src, e_ref, n_tok, dim, ref_last_refresh, cold, bands, g_stamp);

@@ -236,6 +236,18 @@ def test_many_keys_online_softmax_groups(pkg, oracle_mod):
     run_side_by_side(pkg, oracle_mod, shape, w, frames, 16, 2, check_caches=True)
 
 
+@pytest.mark.parametrize("ref_mode", [synth.REF_PREV_FRAME, synth.REF_LAST_REFRESH])
+def test_bulk_copy_gather(pkg, oracle_mod, monkeypatch, ref_mode):
+    # the indexed row gather with its rows staged through shared memory by TMA bulk
+    # copies (the alternative to the direct 128-bit loads) gives the same lists, tokens
+    # and reference caches
+    monkeypatch.setenv("IVIT_GATHER", "tma")
+    shape = SHAPE_C
+    w = synth.make_weights(shape, 143)
+    frames = list(synth.stream_random(shape, 2, 4, 144, change_p=0.3))
+    run_side_by_side(pkg, oracle_mod, shape, w, frames, 1, 2, ref_mode=ref_mode, check_caches=True)
+
+
 def test_frames_at_an_odd_address(pkg, monkeypatch):
     # without graphs the patchify kernel reads the caller's frames directly: frames that
     # start at an odd byte address take its byte-load path and must give the same tokens
