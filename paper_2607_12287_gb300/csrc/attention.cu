@@ -14,7 +14,11 @@
 // with 64 keys per CTA an attention CTA fits on an SM beside a GEMM CTA and starts (and
 // prefetches) while the QKV GEMM is still running.
 //
-// Per item and CTA, 128 threads; thread i <-> query row i <-> TMEM lane i:
+// Per item and CTA, 128 threads (thread i <-> query row i <-> TMEM lane i) or, for key
+// groups of 128 keys and more, 256: threads i and i + 128 share row i, each taking every
+// other 32-key chunk of S (their partial row maxima and sums meet in shared memory) and
+// every other 16-column chunk of the output, so that two warps per TMEM lane quadrant
+// hide each other's latencies:
 //   Q tile [128 rows][dh] by TMA (128-byte swizzle, 64-column slices; the padding columns
 //   dh..round16(dh) are zeroed in shared memory); K, V of the CTA's keys by TMA into
 //   [kpc keys][64 columns] slices;
@@ -50,17 +54,22 @@ constexpr int MAX_SPLITS = 8;
 // Shared-memory and TMEM layout of one CTA for kpc keys and head width dhp (padded to
 // 16), identical on host and device.
 struct AttnLayout {
+  int nt;        // threads per CTA (128 or 256)
   int nsl;       // 64-column slices per row
   int kgrp;      // keys per group: the CTA's keys, at most AKMAX (more run in several groups)
   int kpad;      // keys per group rounded up to 64 (K/V slice rows)
   int kslice;    // bytes of one K or V slice
   int rp, pst;   // merge: row slots per owner, row stride of a partial output (floats)
-  int off_q, off_p, off_k, off_v, off_part, off_bar, bytes;
+  int off_q, off_p, off_k, off_v, off_part, off_red, off_bar, bytes;
   int tm_o, tm_cols;
 };
 
+// Threads per CTA for kpc keys per CTA: two per query row once a key group holds 128 keys.
+__host__ __device__ inline int attn_threads(int kpc) { return kpc >= 128 ? 2 * AQ : AQ; }
+
 __host__ __device__ inline AttnLayout attn_layout(int kpc, int dhp, int ns) {
   AttnLayout L;
+  L.nt = attn_threads(kpc);
   L.nsl = dhp > 64 ? 2 : 1;
   L.kgrp = kpc < AKMAX ? kpc : AKMAX;
   L.kpad = (L.kgrp + 63) / 64 * 64;
@@ -73,7 +82,8 @@ __host__ __device__ inline AttnLayout attn_layout(int kpc, int dhp, int ns) {
   L.off_v = L.off_k + L.nsl * L.kslice;
   L.off_part = L.off_v + L.nsl * L.kslice;
   const int part = ns > 1 ? ns * L.rp * (L.pst + 2) * 4 : 0;  // O_s, m, l of every slot
-  L.off_bar = L.off_part + (part + 1023) / 1024 * 1024;
+  L.off_red = L.off_part + (part + 1023) / 1024 * 1024;
+  L.off_bar = L.off_red + (L.nt > AQ ? 2 * AQ * 4 : 0);  // row max / sum exchange [2][AQ]
   L.bytes = L.off_bar + 64 + 1024;  // barriers + TMEM slot, alignment slack
   L.tm_o = L.kpad;
   int need = L.kpad + dhp, cols = 32;
@@ -112,14 +122,55 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-template <int DHP>
-__global__ void __launch_bounds__(128, 1)
+// Running maximum of the valid entries (index < lim) of a 32-column chunk of S, in four
+// independent accumulators.
+__device__ __forceinline__ void chunk_max(const uint32_t (&r)[32], int lim, float (&mx)[4]) {
+  if (lim >= 32) {
+#pragma unroll
+    for (int u = 0; u < 32; ++u) mx[u & 3] = fmaxf(mx[u & 3], __uint_as_float(r[u]));
+  } else {
+#pragma unroll
+    for (int u = 0; u < 32; ++u)
+      if (u < lim) mx[u & 3] = fmaxf(mx[u & 3], __uint_as_float(r[u]));
+  }
+}
+
+// P = 2^(S c - mo) of a 32-column chunk (0 past lim), rounded to bf16 and stored as the
+// row's 16-byte chunks kc0.. of the P operand (those below gns); lsum gets the rounded
+// values.
+__device__ __forceinline__ void chunk_exp(const uint32_t (&r)[32], int lim, float sc, float mo, uint8_t* sp,
+                                          int row, int kc0, int gns, float (&lsum)[4]) {
+  uint32_t pk[16];
+#pragma unroll
+  for (int u = 0; u < 16; ++u) {
+    const int j = 2 * u;
+    const float p0 = j < lim ? ex2(fmaf(__uint_as_float(r[j]), sc, -mo)) : 0.f;
+    const float p1 = j + 1 < lim ? ex2(fmaf(__uint_as_float(r[j + 1]), sc, -mo)) : 0.f;
+    const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
+    const float2 f = __bfloat1622float2(b);
+    lsum[u & 3] += f.x + f.y;  // the normaliser sums the values the MMA multiplies
+    pk[u] = *reinterpret_cast<const uint32_t*>(&b);
+  }
+#pragma unroll
+  for (int q4 = 0; q4 < 4; ++q4) {
+    const int kc = kc0 + q4;  // 16-byte chunk (8 keys) of this row of P
+    if (kc * 8 < gns)
+      *reinterpret_cast<uint4*>(sp + (kc >> 3) * SLICE_Q + swz(row, kc & 7)) =
+          make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
+  }
+}
+
+template <int DHP, int NT>
+__global__ void __launch_bounds__(NT, 1)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                         const __grid_constant__ CUtensorMap tm_v, const AttnTcArgs a) {
+  constexpr int NH = NT / AQ;                       // threads per query row
+  constexpr int OCH = (DHP / 16 + NH - 1) / NH;     // 16-column output chunks per thread
   extern __shared__ uint8_t at_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(at_raw) + 1023) &
                                            ~static_cast<uintptr_t>(1023));
   const int tid = threadIdx.x, warp = tid >> 5;
+  const int row = tid & (AQ - 1), hf = tid / AQ;  // query row (TMEM lane) and column half
   const int N = a.n_tok, D = a.dim, dh = a.dh;
   const int n_items = a.sv * a.heads * a.qtiles;
   const int ns = static_cast<int>(cluster_nctarank()), rank = static_cast<int>(cluster_ctarank());
@@ -137,6 +188,7 @@ __global__ void __launch_bounds__(128, 1)
   float* po = reinterpret_cast<float*>(sm + L.off_part);
   float* pm = po + ns * L.rp * L.pst;
   float* pl = pm + ns * L.rp;
+  float* red = reinterpret_cast<float*>(sm + L.off_red);  // [NH][AQ] partial row max / sum
 
   // The row offsets come from the selection kernel, at least two launches back (every
   // kernel of the library triggers its dependents only after its own wait).  Every CTA
@@ -165,7 +217,7 @@ __global__ void __launch_bounds__(128, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
-  const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+  const uint32_t trow = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
   const uint32_t tm_s = tmem, tm_o = tmem + static_cast<uint32_t>(L.tm_o);
   const uint64_t pol_q = l2_policy_evict_first(), pol_kv = l2_policy_evict_last();
 
@@ -225,7 +277,7 @@ __global__ void __launch_bounds__(128, 1)
     }
     if (!mbar_wait(bq, ph_q & 1)) ok = false;
     ++ph_q;
-    if (DHP != dh) {  // columns dh..dh+7 of the Q tile hold the next head: zero them
+    if (DHP != dh && tid < AQ) {  // columns dh..dh+7 of the Q tile hold the next head: zero them
       const int c = dh >> 3;
       *reinterpret_cast<uint4*>(sm + L.off_q + (c >> 3) * SLICE_Q + swz(tid, c & 7)) = make_uint4(0, 0, 0, 0);
     }
@@ -235,11 +287,11 @@ __global__ void __launch_bounds__(128, 1)
 
     // Online softmax over the key groups (running max m, running sum l, output in
     // registers rescaled by 2^((m_old - m_new) c) when the max grows).
-    const bool wrow = warp * 32 < it.nq;  // warp-uniform: padding warps skip the math
-    float m_run = -INFINITY, l_run = 0.f;
-    float o_run[DHP];
+    const bool wrow = (warp & 3) * 32 < it.nq;  // warp-uniform: padding warps skip the math
+    float m_run = -INFINITY, l_run = 0.f;       // l_run: this thread's columns only
+    float o_run[OCH * 16];                      // chunks hf, hf + NH, ... of the output row
 #pragma unroll
-    for (int d = 0; d < DHP; ++d) o_run[d] = 0.f;
+    for (int d = 0; d < OCH * 16; ++d) o_run[d] = 0.f;
     for (int g = 0; g < ngroups; ++g) {
       const int gn = min(G, nk - g * G), gns = (gn + 15) & ~15;
       // ---- S = Q K^T
@@ -263,46 +315,62 @@ __global__ void __launch_bounds__(128, 1)
       tc_fence_after();
       if (tid == 0 && g + 1 < ngroups) load_kv(bk, L.off_k, &tm_k, it.v, it.h, g + 1);  // K tile consumed
 
-      // ---- softmax of the group, P to shared memory
+      // ---- softmax of the group, P to shared memory.  This thread's 32-column chunks of
+      // S are cb = 32 hf, 32 (hf + NH), ...; two TMEM loads are in flight at a time.
       float alpha = 1.f;
+      float mpart = -INFINITY;
       if (wrow) {
-        float mc = -INFINITY;
-        for (int cb = 0; cb < gns; cb += 64) {
+        float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        for (int cb = 32 * hf; cb < gns; cb += 64 * NH) {
+          const int cb1 = cb + 32 * NH;
           uint32_t r0[32], r1[32];
           tmem_ld32_async(trow + cb, r0);
-          tmem_ld32_async(trow + cb + 32, r1);
-          tmem_ld_wait();
-#pragma unroll
-          for (int u = 0; u < 32; ++u) {
-            if (cb + u < gn) mc = fmaxf(mc, __uint_as_float(r0[u]));
-            if (cb + 32 + u < gn) mc = fmaxf(mc, __uint_as_float(r1[u]));
+          if (cb1 < gns) tmem_ld32_async(trow + cb1, r1);
+          tmem_ld_wait_regs(r0);
+          chunk_max(r0, gn - cb, mx);
+          if (cb1 < gns) {
+            tmem_ld_wait_regs(r1);
+            chunk_max(r1, gn - cb1, mx);
           }
         }
-        const float m_new = fmaxf(m_run, mc);
+        mpart = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+      }
+      if (NH > 1) {  // the row's maximum over both halves' columns
+        red[hf * AQ + row] = mpart;
+        __syncthreads();
+        mpart = fmaxf(mpart, red[(hf ^ 1) * AQ + row]);
+      }
+      if (wrow) {
+        const float m_new = fmaxf(m_run, mpart);
         alpha = ex2((m_run - m_new) * sc);  // 0 on the first group (m_run = -inf)
         const float mo = m_new * sc;
         float lsum[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int cb = 0; cb < gns; cb += 32) {
-          uint32_t r[32];
-          tmem_ld32_async(trow + cb, r);
-          tmem_ld_wait();
-          uint32_t pk[16];
-#pragma unroll
-          for (int u = 0; u < 16; ++u) {
-            const int j = cb + 2 * u;
-            const float p0 = j < gn ? ex2(fmaf(__uint_as_float(r[2 * u]), sc, -mo)) : 0.f;
-            const float p1 = j + 1 < gn ? ex2(fmaf(__uint_as_float(r[2 * u + 1]), sc, -mo)) : 0.f;
-            const __nv_bfloat162 b = __floats2bfloat162_rn(p0, p1);
-            const float2 f = __bfloat1622float2(b);
-            lsum[u & 3] += f.x + f.y;  // the normaliser sums the values the MMA multiplies
-            pk[u] = *reinterpret_cast<const uint32_t*>(&b);
+        if constexpr (NH > 1) {
+          uint32_t ra[32], rb[32];
+          int cb = 32 * hf;
+          if (cb < gns) {
+            tmem_ld32_async(trow + cb, ra);
+            tmem_ld_wait_regs(ra);
           }
-#pragma unroll
-          for (int q4 = 0; q4 < 4; ++q4) {
-            const int kc = (cb >> 3) + q4;  // 16-byte chunk (8 keys) of this row of P
-            if (kc * 8 < gns)
-              *reinterpret_cast<uint4*>(sm + L.off_p + (kc >> 3) * SLICE_Q + swz(tid, kc & 7)) =
-                  make_uint4(pk[4 * q4], pk[4 * q4 + 1], pk[4 * q4 + 2], pk[4 * q4 + 3]);
+          while (cb < gns) {  // chunk cb is in ra; the next one loads while it is used
+            const int cn = cb + 32 * NH;
+            if (cn < gns) tmem_ld32_async(trow + cn, rb);
+            chunk_exp(ra, gn - cb, sc, mo, sm + L.off_p, row, cb >> 3, gns, lsum);
+            if (cn >= gns) break;
+            tmem_ld_wait_regs(rb);
+            const int cn2 = cn + 32 * NH;
+            if (cn2 < gns) tmem_ld32_async(trow + cn2, ra);
+            chunk_exp(rb, gn - cn, sc, mo, sm + L.off_p, row, cn >> 3, gns, lsum);
+            if (cn2 >= gns) break;
+            tmem_ld_wait_regs(ra);
+            cb = cn2;
+          }
+        } else {  // one thread per row holds the whole output row: one chunk at a time
+          for (int cb = 0; cb < gns; cb += 32) {
+            uint32_t r[32];
+            tmem_ld32_async(trow + cb, r);
+            tmem_ld_wait_regs(r);
+            chunk_exp(r, gn - cb, sc, mo, sm + L.off_p, row, cb >> 3, gns, lsum);
           }
         }
         l_run = l_run * alpha + ((lsum[0] + lsum[1]) + (lsum[2] + lsum[3]));
@@ -336,11 +404,14 @@ __global__ void __launch_bounds__(128, 1)
       if (tid == 0 && g + 1 < ngroups) load_kv(bv, L.off_v, &tm_v, it.v, it.h, g + 1);  // V tile consumed
       if (wrow) {  // warp-uniform: tcgen05.ld is a warp-collective instruction
 #pragma unroll
-        for (int c = 0; c < DHP; c += 16) {
-          float ov[16];
-          tmem_ld16(trow + L.tm_o + c, ov);
+        for (int q = 0; q < OCH; ++q) {
+          const int c = (hf + q * NH) * 16;
+          if (c < DHP) {
+            float ov[16];
+            tmem_ld16(trow + L.tm_o + c, ov);
 #pragma unroll
-          for (int u = 0; u < 16; ++u) o_run[c + u] = o_run[c + u] * alpha + ov[u];
+            for (int u = 0; u < 16; ++u) o_run[q * 16 + u] = o_run[q * 16 + u] * alpha + ov[u];
+          }
         }
       }
     }
@@ -350,21 +421,32 @@ __global__ void __launch_bounds__(128, 1)
     Item nxt;
     while (s_next < n_items && !item_at(s_next, a, nxt)) s_next += ncl;
 
+    if (NH > 1) {  // the row's sum over both halves' columns (the same order on both)
+      red[hf * AQ + row] = l_run;
+      __syncthreads();
+      const float lo_ = red[row], hi_ = red[AQ + row];
+      l_run = lo_ + hi_;
+    }
     if (ns == 1) {
-      if (wrow && tid < it.nq) {
+      if (wrow && row < it.nq) {
         const float inv = 1.f / l_run;
-        bf16* orow = a.o + static_cast<size_t>(it.r0 + tid) * D + it.h * dh;
+        bf16* orow = a.o + static_cast<size_t>(it.r0 + row) * D + it.h * dh;
 #pragma unroll
-        for (int c = 0; c < DHP; c += 8) {
-          if (c < dh) {
-            uint4 u;
-            uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+        for (int q = 0; q < OCH; ++q) {
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const __nv_bfloat162 b = __floats2bfloat162_rn(o_run[c + 2 * e] * inv, o_run[c + 2 * e + 1] * inv);
-              w[e] = *reinterpret_cast<const uint32_t*>(&b);
+          for (int h8 = 0; h8 < 16; h8 += 8) {
+            const int c = (hf + q * NH) * 16 + h8;
+            if (c < dh) {
+              uint4 u;
+              uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const __nv_bfloat162 b = __floats2bfloat162_rn(o_run[q * 16 + h8 + 2 * e] * inv,
+                                                               o_run[q * 16 + h8 + 2 * e + 1] * inv);
+                w[e] = *reinterpret_cast<const uint32_t*>(&b);
+              }
+              *reinterpret_cast<uint4*>(orow + c) = u;
             }
-            *reinterpret_cast<uint4*>(orow + c) = u;
           }
         }
       }
@@ -372,15 +454,24 @@ __global__ void __launch_bounds__(128, 1)
       // push this CTA's partial (m, l, O_s) of row i to slot [rank][i - owner * rpi] of
       // the owner CTA i / rpi; a CTA without keys pushes m = -inf, l = 0, O = 0
       const int rpi = (it.nq + ns - 1) / ns;  // rows per owner in this item (<= rp)
-      if (tid < it.nq) {
-        const int owner = tid / rpi, slot = tid - owner * rpi;
+      if (row < it.nq) {
+        const int owner = row / rpi, slot = row - owner * rpi;
         const uint32_t obase =
             mapa_shared(smem_u32(po + (rank * L.rp + slot) * L.pst), static_cast<uint32_t>(owner));
 #pragma unroll
-        for (int c = 0; c < DHP; c += 4)
-          st_dsmem_f32x4(obase + 4 * c, make_float4(o_run[c], o_run[c + 1], o_run[c + 2], o_run[c + 3]));
-        st_dsmem_f32(mapa_shared(smem_u32(pm + rank * L.rp + slot), static_cast<uint32_t>(owner)), m_run);
-        st_dsmem_f32(mapa_shared(smem_u32(pl + rank * L.rp + slot), static_cast<uint32_t>(owner)), l_run);
+        for (int q = 0; q < OCH; ++q) {
+          const int c0 = (hf + q * NH) * 16;
+          if (c0 < DHP) {
+#pragma unroll
+            for (int c = 0; c < 16; c += 4)
+              st_dsmem_f32x4(obase + 4 * (c0 + c), make_float4(o_run[q * 16 + c], o_run[q * 16 + c + 1],
+                                                               o_run[q * 16 + c + 2], o_run[q * 16 + c + 3]));
+          }
+        }
+        if (hf == 0) {
+          st_dsmem_f32(mapa_shared(smem_u32(pm + rank * L.rp + slot), static_cast<uint32_t>(owner)), m_run);
+          st_dsmem_f32(mapa_shared(smem_u32(pl + rank * L.rp + slot), static_cast<uint32_t>(owner)), l_run);
+        }
       }
       cluster_sync();  // every rank's partials of this CTA's rows are in its shared memory
       const int lo = rank * rpi, nmine = max(0, min(it.nq, lo + rpi) - lo);
@@ -440,8 +531,11 @@ __global__ void __launch_bounds__(128, 1)
 
 template <int DHP>
 cudaError_t launch_dhp(const CUtensorMap& tm_q, const CUtensorMap& tm_k, const CUtensorMap& tm_v,
-                       const AttnTcArgs& a, int grid, int smem, cudaStream_t s) {
-  return launch_ex(attention_tc_kernel<DHP>, dim3(grid), dim3(128), static_cast<size_t>(smem), s,
+                       const AttnTcArgs& a, int grid, int smem, int nt, cudaStream_t s) {
+  if (nt > AQ)
+    return launch_ex(attention_tc_kernel<DHP, 2 * AQ>, dim3(grid), dim3(nt), static_cast<size_t>(smem), s,
+                     static_cast<unsigned>(a.key_splits), tm_q, tm_k, tm_v, a);
+  return launch_ex(attention_tc_kernel<DHP, AQ>, dim3(grid), dim3(nt), static_cast<size_t>(smem), s,
                    static_cast<unsigned>(a.key_splits), tm_q, tm_k, tm_v, a);
 }
 
@@ -469,14 +563,22 @@ cudaError_t attention_tc_setup() {
   auto set = [&](auto kern) {
     if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, max_bytes);
   };
-  set(attention_tc_kernel<16>);
-  set(attention_tc_kernel<32>);
-  set(attention_tc_kernel<48>);
-  set(attention_tc_kernel<64>);
-  set(attention_tc_kernel<80>);
-  set(attention_tc_kernel<96>);
-  set(attention_tc_kernel<112>);
-  set(attention_tc_kernel<128>);
+  set(attention_tc_kernel<16, AQ>);
+  set(attention_tc_kernel<16, 2 * AQ>);
+  set(attention_tc_kernel<32, AQ>);
+  set(attention_tc_kernel<32, 2 * AQ>);
+  set(attention_tc_kernel<48, AQ>);
+  set(attention_tc_kernel<48, 2 * AQ>);
+  set(attention_tc_kernel<64, AQ>);
+  set(attention_tc_kernel<64, 2 * AQ>);
+  set(attention_tc_kernel<80, AQ>);
+  set(attention_tc_kernel<80, 2 * AQ>);
+  set(attention_tc_kernel<96, AQ>);
+  set(attention_tc_kernel<96, 2 * AQ>);
+  set(attention_tc_kernel<112, AQ>);
+  set(attention_tc_kernel<112, 2 * AQ>);
+  set(attention_tc_kernel<128, AQ>);
+  set(attention_tc_kernel<128, 2 * AQ>);
   return e;
 }
 
@@ -489,15 +591,16 @@ cudaError_t launch_attention_tc(const CUtensorMap& tm_q, const CUtensorMap& tm_k
   const int grid = clusters * ns;
   const int smem = static_cast<int>(attention_tc_smem(a.n_tok, a.dh, ns));
   if (smem > smem_optin()) return cudaErrorInvalidValue;
+  const int nt = attn_threads((a.n_tok + ns - 1) / ns);
   switch ((a.dh + 15) & ~15) {
-    case 16: return launch_dhp<16>(tm_q, tm_k, tm_v, a, grid, smem, s);
-    case 32: return launch_dhp<32>(tm_q, tm_k, tm_v, a, grid, smem, s);
-    case 48: return launch_dhp<48>(tm_q, tm_k, tm_v, a, grid, smem, s);
-    case 64: return launch_dhp<64>(tm_q, tm_k, tm_v, a, grid, smem, s);
-    case 80: return launch_dhp<80>(tm_q, tm_k, tm_v, a, grid, smem, s);
-    case 96: return launch_dhp<96>(tm_q, tm_k, tm_v, a, grid, smem, s);
-    case 112: return launch_dhp<112>(tm_q, tm_k, tm_v, a, grid, smem, s);
-    case 128: return launch_dhp<128>(tm_q, tm_k, tm_v, a, grid, smem, s);
+    case 16: return launch_dhp<16>(tm_q, tm_k, tm_v, a, grid, smem, nt, s);
+    case 32: return launch_dhp<32>(tm_q, tm_k, tm_v, a, grid, smem, nt, s);
+    case 48: return launch_dhp<48>(tm_q, tm_k, tm_v, a, grid, smem, nt, s);
+    case 64: return launch_dhp<64>(tm_q, tm_k, tm_v, a, grid, smem, nt, s);
+    case 80: return launch_dhp<80>(tm_q, tm_k, tm_v, a, grid, smem, nt, s);
+    case 96: return launch_dhp<96>(tm_q, tm_k, tm_v, a, grid, smem, nt, s);
+    case 112: return launch_dhp<112>(tm_q, tm_k, tm_v, a, grid, smem, nt, s);
+    case 128: return launch_dhp<128>(tm_q, tm_k, tm_v, a, grid, smem, nt, s);
     default: return cudaErrorInvalidValue;
   }
 }

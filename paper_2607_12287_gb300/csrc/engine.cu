@@ -519,6 +519,7 @@ int setup(ivit_handle* h, const uint16_t* wb) {
       const int ns_cap = std::max(1, std::min(8, (h->N + 63) / 64));  // at least 64 keys per CTA
       const int items = h->SV * h->H * ((m_exp + 127) / 128);
       int ns = std::max(1, std::min(ns_cap, h->num_sms / std::max(1, items)));
+      if (const char* e = std::getenv("IVIT_ATTN_SPLITS")) ns = std::max(1, std::min(8, std::atoi(e)));
       while (ns < 8 && ivit::attention_tc_smem(h->N, dh, ns) > static_cast<size_t>(optin)) ++ns;
       return ns;
     };
