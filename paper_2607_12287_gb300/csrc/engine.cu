@@ -42,6 +42,7 @@ struct TimelineSlot {
 // Launch shape of one GEMM: row-tile variant, CTAs per cluster (the K split), clusters.
 struct GemmPlan {
   int bn = 64, csize = 1, n_clusters = 1;
+  bool defer = false;  // residual GEMMs: leave the split partials to the next layer norm
 };
 
 enum GemmSlot { kGemmEmbed = 0, kGemmQKV, kGemmO, kGemmUp, kGemmDown, kGemmSlots };
@@ -554,6 +555,20 @@ int setup(ivit_handle* h, const uint16_t* wb) {
                                              : plan_gemm(h->num_sms, h->band_ub[b] <= 64 ? 64 : 256, shapes[g][0],
                                                          shapes[g][1], h->band_ub[b]);
     }
+    // Residual GEMMs split over clusters leave their partials to the layer norm that
+    // follows (one slot per tile and split, sized for the most rows the plan can see),
+    // while that scratch stays under 64 MB.
+    auto set_defer = [&](GemmPlan& pl, int n_out, int m_bound) {
+      const size_t slots = static_cast<size_t>((n_out + 127) / 128) * ((m_bound + pl.bn - 1) / pl.bn) * pl.csize;
+      pl.defer = pl.csize > 1 && !std::getenv("IVIT_NO_DEFER") && slots * pl.bn * 128 * 4 <= (64ull << 20) &&
+                 h->D % 4 == 0 && h->D <= 4096;
+    };
+    for (int g : {static_cast<int>(kGemmO), static_cast<int>(kGemmDown)}) {
+      set_defer(h->plan_full[g], static_cast<int>(D), static_cast<int>(M));
+      set_defer(h->plan_inc[g], static_cast<int>(D), static_cast<int>(M));
+      h->plan_band[0][g] = h->plan_inc[g];
+      for (int b = 1; b < h->n_bands; ++b) set_defer(h->plan_band[b][g], static_cast<int>(D), h->band_ub[b]);
+    }
     if (std::getenv("IVIT_DEBUG")) {
       static const char* names[kGemmSlots] = {"embed", "qkv", "out", "up", "down"};
       for (int g = 0; g < kGemmSlots; ++g)
@@ -662,12 +677,14 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   size_t part_floats = 0;
   for (int g = 0; g < kGemmSlots; ++g)
   {
-    for (const GemmPlan* pl : {&h->plan_full[g], &h->plan_inc[g]})
-      part_floats = std::max(part_floats, static_cast<size_t>(pl->n_clusters) * pl->csize * pl->bn * 128);
-    for (int b = 0; b < h->n_bands; ++b) {
-      const GemmPlan& pl = h->plan_band[b][g];
-      part_floats = std::max(part_floats, static_cast<size_t>(pl.n_clusters) * pl.csize * pl.bn * 128);
-    }
+    auto need = [&](const GemmPlan& pl, int m_bound) {
+      if (!pl.defer) return static_cast<size_t>(pl.n_clusters) * pl.csize * pl.bn * 128;
+      return static_cast<size_t>((D + 127) / 128) * ((m_bound + pl.bn - 1) / pl.bn) * pl.csize * pl.bn * 128;
+    };
+    part_floats = std::max(part_floats, need(h->plan_full[g], static_cast<int>(M)));
+    part_floats = std::max(part_floats, need(h->plan_inc[g], static_cast<int>(M)));
+    for (int b = 0; b < h->n_bands; ++b)
+      part_floats = std::max(part_floats, need(h->plan_band[b][g], b == 0 ? static_cast<int>(M) : h->band_ub[b]));
   }
   const size_t o_gpart = sa.take(part_floats * 4);
   const size_t o_rta = sa.take(M * 4), o_mall = sa.take(4);
@@ -988,14 +1005,46 @@ int run_layers(ivit_handle* h, const GemmPlan* plan, int attn_splits, bool full,
   const ivit_config& c = h->cfg;
   const int D = h->D, F = h->F, SV = h->SV, M = h->M_max;
   const int* total = h->cu_rows + SV;
+  // A residual update still split over the GEMM scratch (deferred out-projection or
+  // MLP-down GEMM): the next layer norm adds it to x.
+  ivit::PendingSum pend;
+  auto layernorm = [&](const float* g, const float* b, bf16* y, const int* dst) -> int {
+    next_launch(h, kFamLN);
+    if (pend.partials) {
+      IVIT_CK(h, ivit::launch_layernorm_sum(total, h->x, pend, g, b, y, dst, D, c.ln_eps, M, h->row_grid, s));
+      pend = ivit::PendingSum();
+    } else {
+      IVIT_CK(h, ivit::launch_layernorm(total, h->x, g, b, y, dst, D, c.ln_eps, M, h->row_grid, s));
+    }
+    ++h->launches;
+    return IVIT_OK;
+  };
+  auto residual = [&](const GemmPlan& pl, const float* bias, const CUtensorMap& tw, const CUtensorMap& tx,
+                      int k) -> int {
+    ivit::GemmArgs a;
+    a.n_out = D;
+    a.k = k;
+    a.d_rows = total;
+    a.epi.kind = ivit::kEpiResid;
+    a.epi.bias = bias;
+    a.epi.out_f32 = h->x;
+    a.epi.ld_out = D;
+    a.defer = pl.defer ? 1 : 0;
+    if (int r = gemm(h, pl, tw, tx, a, s)) return r;
+    if (pl.defer) {
+      pend.partials = h->gemm_partials;
+      pend.bias = bias;
+      pend.csize = pl.csize;
+      pend.bn = pl.bn;
+      pend.n_ft = (D + 127) / 128;
+    }
+    return IVIT_OK;
+  };
   for (int l = 0; l < h->L; ++l) {
     const LayerW& w = h->layers[l];
     bf16* ck = h->cacheK + static_cast<size_t>(l) * M * D;
     bf16* cv = h->cacheV + static_cast<size_t>(l) * M * D;
-    next_launch(h, kFamLN);
-    IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln1g, w.ln1b, h->xn, nullptr, D, c.ln_eps, M,
-                                      h->row_grid, s));
-    ++h->launches;
+    if (int r = layernorm(w.ln1g, w.ln1b, h->xn, nullptr)) return r;
     {
       ivit::GemmArgs a;
       a.n_out = 3 * D;
@@ -1012,21 +1061,8 @@ int run_layers(ivit_handle* h, const GemmPlan* plan, int attn_splits, bool full,
       if (int r = gemm(h, plan[kGemmQKV], w.tm_qkv, h->tm_xn, a, s)) return r;
     }
     if (int r = attention(h, w, ck, cv, full, s, attn_splits)) return r;
-    {
-      ivit::GemmArgs a;
-      a.n_out = D;
-      a.k = D;
-      a.d_rows = total;
-      a.epi.kind = ivit::kEpiResid;
-      a.epi.bias = w.bo;
-      a.epi.out_f32 = h->x;
-      a.epi.ld_out = D;
-      if (int r = gemm(h, plan[kGemmO], w.tm_o, h->tm_o, a, s)) return r;
-    }
-    next_launch(h, kFamLN);
-    IVIT_CK(h, ivit::launch_layernorm(total, h->x, w.ln2g, w.ln2b, h->xn, nullptr, D, c.ln_eps, M,
-                                      h->row_grid, s));
-    ++h->launches;
+    if (int r = residual(plan[kGemmO], w.bo, w.tm_o, h->tm_o, D)) return r;
+    if (int r = layernorm(w.ln2g, w.ln2b, h->xn, nullptr)) return r;
     {
       ivit::GemmArgs a;
       a.n_out = F;
@@ -1039,23 +1075,9 @@ int run_layers(ivit_handle* h, const GemmPlan* plan, int attn_splits, bool full,
       a.epi.gelu_mode = c.gelu;
       if (int r = gemm(h, plan[kGemmUp], w.tm_1, h->tm_xn, a, s)) return r;
     }
-    {
-      ivit::GemmArgs a;
-      a.n_out = D;
-      a.k = F;
-      a.d_rows = total;
-      a.epi.kind = ivit::kEpiResid;
-      a.epi.bias = w.b2;
-      a.epi.out_f32 = h->x;
-      a.epi.ld_out = D;
-      if (int r = gemm(h, plan[kGemmDown], w.tm_2, h->tm_h, a, s)) return r;
-    }
+    if (int r = residual(plan[kGemmDown], w.b2, w.tm_2, h->tm_h, F)) return r;
   }
-  next_launch(h, kFamLN);
-  IVIT_CK(h, ivit::launch_layernorm(total, h->x, h->lnfg, h->lnfb, h->tok_out, h->rowtok, D, c.ln_eps,
-                                    M, h->row_grid, s));
-  ++h->launches;
-  return IVIT_OK;
+  return layernorm(h->lnfg, h->lnfb, h->tok_out, h->rowtok);
 }
 
 // Under capture of an incremental graph with row bands: a switch node after the
@@ -1094,7 +1116,7 @@ int capture_band_bodies(ivit_handle* h, cudaStream_t s) {
 // Enqueues the whole chain for one frame per view on `s` (eagerly or under capture).
 int run_core(ivit_handle* h, const uint8_t* frames, int32_t* user_counts, bool full, cudaStream_t s) {
   const ivit_config& c = h->cfg;
-  const int N = h->N, D = h->D, F = h->F, SV = h->SV, M = h->M_max;
+  const int N = h->N, D = h->D, SV = h->SV, M = h->M_max;
   ivit::ColdMask cm;
   std::memset(&cm, 0, sizeof cm);
   for (int v = 0; v < SV; ++v)

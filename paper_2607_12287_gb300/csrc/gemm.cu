@@ -13,7 +13,10 @@
 // writes its fp32 partial tile from TMEM to its slot of a global scratch (it stays in
 // L2), and after a cluster barrier every CTA sums a slice of the tile's rows over all
 // slots, in rank order (deterministic), and runs the epilogue.  The scratch outlives
-// the CTAs, so a cluster with no further tile leaves without a second barrier.
+// the CTAs, so a cluster with no further tile leaves without a second barrier.  A
+// deferred launch (residual epilogue, small row counts) stops after writing its partial
+// tile, into a slot of its own per tile: the layer norm that follows sums the slots, so
+// neither the cluster barrier nor the reduction sits on this kernel's critical path.
 // Clusters walk the output tiles (feature tile x row tile) with a stride.
 //
 // Pipeline per CTA (128 threads): warp 0 lane 0 issues TMA loads (weights with an
@@ -254,7 +257,8 @@ __global__ void __launch_bounds__(128, 1)
       // of the tile's rows over all slots in rank order.  Global memory outlives the CTA,
       // so only a following tile of this cluster (which reuses the slots) needs a second
       // barrier.
-      float* mine = a.partials + static_cast<size_t>(cl_id * csize + crank) * BN_MAX * BM;
+      const int slot = a.defer ? tile * csize + crank : cl_id * csize + crank;
+      float* mine = a.partials + static_cast<size_t>(slot) * BN_MAX * BM;
       if (ok && has_k) {
         for (int c0 = 0; c0 < rows; c0 += 16) {
           float v[16];
@@ -265,6 +269,11 @@ __global__ void __launch_bounds__(128, 1)
         }
       } else {
         for (int c = 0; c < rows; ++c) mine[c * BM + fl] = 0.f;
+      }
+      if (a.defer) {  // the next kernel sums the slots: no barrier, no epilogue here
+        tc_fence_before();
+        __syncthreads();  // TMEM is read before the next tile's MMAs
+        continue;
       }
       cluster_sync();  // every partial of this tile is in the scratch
       if (ok) {

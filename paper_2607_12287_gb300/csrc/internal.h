@@ -82,8 +82,24 @@ struct GemmArgs {
   // floats for every CTA of the launch.  Required when the launch's clusters have more
   // than one CTA.
   float* partials = nullptr;
+  // With clusters of more than one CTA and defer set, the split-K partial tiles are left
+  // in the scratch, slot (tile * csize + rank) with tile = feature tile + n_ft * row tile,
+  // and the kernel neither reduces them nor runs the epilogue: the next kernel sums them
+  // (layernorm_sum, for the residual epilogue).  The scratch then holds
+  // n_ft * ceil(M / BN_MAX) * csize slots.
+  int defer = 0;
   unsigned long long* stamp = nullptr;  // timeline stamps of this launch (or null)
   GemmEpilogue epi;
+};
+
+// A residual update x += bias + sum_s partial_s still split over the scratch slots of a
+// deferred GEMM (see GemmArgs::defer).
+struct PendingSum {
+  const float* partials = nullptr;  // the GEMM's scratch
+  const float* bias = nullptr;      // [dim]
+  int csize = 0;                    // splits (CTAs per cluster), 2..16
+  int bn = 0;                       // rows per row tile (the GEMM's BN_MAX)
+  int n_ft = 0;                     // feature tiles of 128
 };
 
 // Returns the dynamic shared memory size (bytes) of the GEMM variant.
@@ -216,6 +232,13 @@ cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma
 cudaError_t launch_layernorm_ex(const int* rows, float* x, const float* add, const int* src_rowtok,
                                 const float* gamma, const float* beta, bf16* y, const int* dst_rowtok, int dim,
                                 float eps, int max_rows, int grid, cudaStream_t s);
+
+// x[r] += bias + sum_s partial_s[r] (splits in order, as the GEMM's own reduction sums
+// them), written back to x, then y = LN(x[r]) (row dst_rowtok[r] of y when set), for
+// r < *rows.  dim a multiple of 4, at most 4096.
+cudaError_t launch_layernorm_sum(const int* rows, float* x, const PendingSum& ps, const float* gamma,
+                                 const float* beta, bf16* y, const int* dst_rowtok, int dim, float eps,
+                                 int max_rows, int grid, cudaStream_t s);
 
 // One-time function attributes of the attention kernel (dynamic shared memory opt-in).
 cudaError_t attention_setup();

@@ -382,6 +382,83 @@ __global__ void layernorm_kernel(const int* __restrict__ nrows, float* __restric
   stamp_end(stamp);
 }
 
+// Layer norm after a deferred split-K GEMM with the residual epilogue: per row, x +=
+// bias + sum_s partial_s (the splits in order, the same fp32 sum the GEMM's own
+// reduction forms), x written back, then y = LN(x).  One CTA per row and one float4 of
+// the row per thread, so every split's partial of every element is in flight at once
+// (a row's partials are spread over the csize slots of its feature tiles).
+__global__ void layernorm_sum_kernel(const int* __restrict__ nrows, float* __restrict__ x, const PendingSum ps,
+                                     const float* __restrict__ gamma, const float* __restrict__ beta,
+                                     bf16* __restrict__ y, const int* __restrict__ dst_rowtok, int dim, float eps,
+                                     unsigned long long* stamp) {
+  constexpr int MAXS = 16;
+  __shared__ float red[2][32];
+  const int c = threadIdx.x;  // float4 of the row
+  const int n4 = dim / 4, lane = c & 31, warp = c >> 5, nw = blockDim.x >> 5;
+  const bool act = c < n4;
+  float4 g = make_float4(0.f, 0.f, 0.f, 0.f), b = g, bias = g;
+  if (act) {  // constants: before the wait on the previous kernel
+    g = reinterpret_cast<const float4*>(gamma)[c];
+    b = reinterpret_cast<const float4*>(beta)[c];
+    bias = reinterpret_cast<const float4*>(ps.bias)[c];
+  }
+  const int rows = *nrows;  // written by the selection kernel, at least two launches back
+  pdl_wait();
+  pdl_launch_dependents();
+  stamp_begin(stamp);
+  const int f = 4 * c, ft = f >> 7, fl = f & 127;
+  const size_t sstride = static_cast<size_t>(ps.bn) * 128;
+  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (act) {
+      const int tt = r / ps.bn, rr = r - tt * ps.bn;
+      const float* p = ps.partials + (static_cast<size_t>(ft + ps.n_ft * tt) * ps.csize * ps.bn + rr) * 128 + fl;
+      float4 q[MAXS];
+#pragma unroll
+      for (int sp = 0; sp < MAXS; ++sp)
+        if (sp < ps.csize) q[sp] = __ldcg(reinterpret_cast<const float4*>(p + sp * sstride));
+      float4* xr = reinterpret_cast<float4*>(x + static_cast<size_t>(r) * dim) + c;
+      const float4 x0 = *xr;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int sp = 0; sp < MAXS; ++sp)
+        if (sp < ps.csize) {
+          acc.x += q[sp].x;
+          acc.y += q[sp].y;
+          acc.z += q[sp].z;
+          acc.w += q[sp].w;
+        }
+      v = make_float4(x0.x + (acc.x + bias.x), x0.y + (acc.y + bias.y), x0.z + (acc.z + bias.z),
+                      x0.w + (acc.w + bias.w));
+      *xr = v;
+    }
+    float sum = warp_sum((v.x + v.y) + (v.z + v.w));
+    if (lane == 0) red[0][warp] = sum;
+    __syncthreads();
+    sum = 0.f;
+    for (int w = 0; w < nw; ++w) sum += red[0][w];
+    const float mean = sum / dim;
+    float sq = 0.f;
+    if (act) {
+      const float a0 = v.x - mean, a1 = v.y - mean, a2 = v.z - mean, a3 = v.w - mean;
+      sq = (a0 * a0 + a1 * a1) + (a2 * a2 + a3 * a3);
+    }
+    sq = warp_sum(sq);
+    if (lane == 0) red[1][warp] = sq;
+    __syncthreads();
+    sq = 0.f;
+    for (int w = 0; w < nw; ++w) sq += red[1][w];
+    const float rstd = rsqrtf(sq / dim + eps);
+    if (act) {
+      const size_t orow = dst_rowtok ? static_cast<size_t>(dst_rowtok[r]) : static_cast<size_t>(r);
+      __nv_bfloat162* yr = reinterpret_cast<__nv_bfloat162*>(y + orow * dim);
+      yr[2 * c] = __floats2bfloat162_rn(g.x * (v.x - mean) * rstd + b.x, g.y * (v.y - mean) * rstd + b.y);
+      yr[2 * c + 1] = __floats2bfloat162_rn(g.z * (v.z - mean) * rstd + b.z, g.w * (v.w - mean) * rstd + b.w);
+    }
+  }
+  stamp_end(stamp);
+}
+
 // -------------------------------------------------------------------- attention
 // Attention of the updated queries of one view over all N keys of that view (cached
 // K/V with this call's updated rows already written), per head:
@@ -655,6 +732,17 @@ cudaError_t launch_layernorm(const int* rows, const float* x, const float* gamma
                              int grid, cudaStream_t s) {
   return launch_layernorm_ex(rows, const_cast<float*>(x), nullptr, nullptr, gamma, beta, y, dst_rowtok, dim, eps,
                              max_rows, grid, s);
+}
+
+cudaError_t launch_layernorm_sum(const int* rows, float* x, const PendingSum& ps, const float* gamma,
+                                 const float* beta, bf16* y, const int* dst_rowtok, int dim, float eps,
+                                 int max_rows, int grid, cudaStream_t s) {
+  if (dim % 4 != 0 || dim > 4096 || ps.csize < 2 || ps.csize > 16 || ps.bn < 1 || !ps.partials || !ps.bias)
+    return cudaErrorInvalidValue;
+  const int threads = (dim / 4 + 31) / 32 * 32;
+  grid = max(1, min(grid, max_rows));
+  return launch_ex(layernorm_sum_kernel, dim3(grid), dim3(threads), 0, s, 1, rows, x, ps, gamma, beta, y,
+                   dst_rowtok, dim, eps, g_stamp);
 }
 
 cudaError_t launch_layernorm_ex(const int* rows, float* x, const float* add, const int* src_rowtok,
