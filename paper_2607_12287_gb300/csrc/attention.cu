@@ -404,13 +404,21 @@ __global__ void __launch_bounds__(NT, 1)
       if (tid == 0 && g + 1 < ngroups) load_kv(bv, L.off_v, &tm_v, it.v, it.h, g + 1);  // V tile consumed
       if (wrow) {  // warp-uniform: tcgen05.ld is a warp-collective instruction
 #pragma unroll
-        for (int q = 0; q < OCH; ++q) {
-          const int c = (hf + q * NH) * 16;
-          if (c < DHP) {
-            float ov[16];
-            tmem_ld16(trow + L.tm_o + c, ov);
+        for (int q = 0; q < OCH; q += 2) {  // two chunks' loads in flight per wait
+          uint32_t ov[2][16];
 #pragma unroll
-            for (int u = 0; u < 16; ++u) o_run[q * 16 + u] = o_run[q * 16 + u] * alpha + ov[u];
+          for (int t = 0; t < 2; ++t)
+            if (q + t < OCH && (hf + (q + t) * NH) * 16 < DHP)
+              tmem_ld16_async(trow + L.tm_o + (hf + (q + t) * NH) * 16, ov[t]);
+          tmem_ld_wait();
+#pragma unroll
+          for (int t = 0; t < 2; ++t) {
+            tmem_regs_after_wait16(ov[t]);
+            if (q + t < OCH && (hf + (q + t) * NH) * 16 < DHP) {
+#pragma unroll
+              for (int u = 0; u < 16; ++u)
+                o_run[(q + t) * 16 + u] = o_run[(q + t) * 16 + u] * alpha + __uint_as_float(ov[t][u]);
+            }
           }
         }
       }

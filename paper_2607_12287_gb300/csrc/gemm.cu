@@ -42,6 +42,9 @@ struct GemmSmem {
   static constexpr int STAGE_BYTES = W_TILE_BYTES + X_TILE_BYTES;
   static constexpr int BAR_OFFSET = STAGES * STAGE_BYTES;
   static constexpr int TOTAL = BAR_OFFSET + 256 + 1024;  // barriers, flags, 1 KB alignment slack
+  // the split-K reduction stages at most (BN_MAX + MAX_CLUSTER) rows of partials, and the
+  // rows' token indices, in the stage memory
+  static_assert((BN_MAX + MAX_CLUSTER) * 128 * 4 + (BN_MAX / 2 + 4) * 4 <= BAR_OFFSET, "reduction staging");
 };
 
 // Hardware tanh (one MUFU instruction, relative error about 2^-11: below the bf16
@@ -58,32 +61,98 @@ __device__ __forceinline__ float gelu_f(float x, int mode) {
   return 0.5f * x * (1.f + tanh_hw(c * (x + 0.044715f * x * x * x)));
 }
 
-__device__ __forceinline__ void epilogue_store(const GemmEpilogue& e, int r, int f, float y) {
-  const float val = y + e.bias[f];
+// Output feature f of TMEM-drained row r; `bias` is bias[f], loaded while the MMAs run.
+// `tok` is rowtok[r] for the epilogues that scatter by token (QKV keys/values,
+// kEpiScatterF32), loaded by the caller together with its other loads; `old` is the
+// residual stream's current value (kEpiResid), likewise.
+__device__ __forceinline__ void epilogue_store(const GemmEpilogue& e, int r, int f, float y, float bias, int tok,
+                                               float old) {
+  const float val = y + bias;
   switch (e.kind) {
     case kEpiF32Bias:
       e.out_f32[static_cast<size_t>(r) * e.ld_out + f] = val;
       break;
     case kEpiResid:
-      e.out_f32[static_cast<size_t>(r) * e.ld_out + f] += val;
+      e.out_f32[static_cast<size_t>(r) * e.ld_out + f] = old + val;
       break;
     case kEpiGelu:
       e.out_bf16[static_cast<size_t>(r) * e.ld_out + f] = __float2bfloat16_rn(gelu_f(val, e.gelu_mode));
       break;
     case kEpiScatterF32:
-      e.out_f32[static_cast<size_t>(e.rowtok[r]) * e.ld_out + f] = val;
+      e.out_f32[static_cast<size_t>(tok) * e.ld_out + f] = val;
       break;
     default: {  // kEpiQKV
       const int D = e.dim;
       if (f < D) {
         e.out_bf16[static_cast<size_t>(r) * e.ld_out + f] = __float2bfloat16_rn(val);
+      } else if (f < 2 * D) {
+        e.cache_k[static_cast<size_t>(tok) * D + (f - D)] = __float2bfloat16_rn(val);
       } else {
-        const size_t tok = static_cast<size_t>(e.rowtok[r]);
-        if (f < 2 * D)
-          e.cache_k[tok * D + (f - D)] = __float2bfloat16_rn(val);
-        else
-          e.cache_v[tok * D + (f - 2 * D)] = __float2bfloat16_rn(val);
+        e.cache_v[static_cast<size_t>(tok) * D + (f - 2 * D)] = __float2bfloat16_rn(val);
       }
+    }
+  }
+}
+
+__device__ __forceinline__ bool epi_needs_tok(int kind) { return kind == kEpiQKV || kind == kEpiScatterF32; }
+
+// One column (output feature f) of up to 16 consecutive rows r0 + j (j < n) drained from
+// TMEM.  Every global load the epilogue needs (row -> token map, residual values) is
+// issued for all 16 rows before the first store, so the rows cost one memory round trip,
+// not one each.
+__device__ __forceinline__ void epilogue_column16(const GemmEpilogue& e, int r0, int n, int f, float bias,
+                                                  const float (&v)[16]) {
+  int tok[16];
+  float old[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    tok[j] = 0;
+    old[j] = 0.f;
+    if (j < n) {
+      if (epi_needs_tok(e.kind)) tok[j] = __ldcg(e.rowtok + r0 + j);
+      if (e.kind == kEpiResid) old[j] = __ldcg(e.out_f32 + static_cast<size_t>(r0 + j) * e.ld_out + f);
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 16; ++j)
+    if (j < n) epilogue_store(e, r0 + j, f, v[j], bias, tok[j], old[j]);
+}
+
+// Four consecutive output features f4..f4+3 (f4 % 4 == 0, all below n_out: every n_out
+// the engine uses is a multiple of 4) of row r, with 8- or 16-byte stores; the bias `b`,
+// `tok` and the residual's current value `o` as in epilogue_store.
+__device__ __forceinline__ void epilogue_store4(const GemmEpilogue& e, int r, int f4, float4 y, float4 b, int tok,
+                                               float4 o) {
+  float4 val = make_float4(y.x + b.x, y.y + b.y, y.z + b.z, y.w + b.w);
+  auto pack4 = [](float4 u) {
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(u.x, u.y), hi = __floats2bfloat162_rn(u.z, u.w);
+    uint2 p;
+    p.x = *reinterpret_cast<const uint32_t*>(&lo);
+    p.y = *reinterpret_cast<const uint32_t*>(&hi);
+    return p;
+  };
+  switch (e.kind) {
+    case kEpiF32Bias:
+      *reinterpret_cast<float4*>(e.out_f32 + static_cast<size_t>(r) * e.ld_out + f4) = val;
+      break;
+    case kEpiResid:
+      *reinterpret_cast<float4*>(e.out_f32 + static_cast<size_t>(r) * e.ld_out + f4) =
+          make_float4(o.x + val.x, o.y + val.y, o.z + val.z, o.w + val.w);
+      break;
+    case kEpiGelu:
+      val = make_float4(gelu_f(val.x, e.gelu_mode), gelu_f(val.y, e.gelu_mode), gelu_f(val.z, e.gelu_mode),
+                        gelu_f(val.w, e.gelu_mode));
+      *reinterpret_cast<uint2*>(e.out_bf16 + static_cast<size_t>(r) * e.ld_out + f4) = pack4(val);
+      break;
+    case kEpiScatterF32:
+      *reinterpret_cast<float4*>(e.out_f32 + static_cast<size_t>(tok) * e.ld_out + f4) = val;
+      break;
+    default: {  // kEpiQKV (D % 4 == 0: the four features lie in one of Q, K, V)
+      const int D = e.dim;
+      bf16* dst = f4 < D ? e.out_bf16 + static_cast<size_t>(r) * e.ld_out + f4
+                         : (f4 < 2 * D ? e.cache_k + static_cast<size_t>(tok) * D + (f4 - D)
+                                       : e.cache_v + static_cast<size_t>(tok) * D + (f4 - 2 * D));
+      *reinterpret_cast<uint2*>(dst) = pack4(val);
     }
   }
 }
@@ -99,12 +168,16 @@ __global__ void __launch_bounds__(128, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::BAR_OFFSET);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 1);
   volatile int* sh_abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  // split-K reduction: row -> token indices of this CTA's rows (at most BN_MAX / 2 + 1)
+  int* red_tok = reinterpret_cast<int*>(smem + L::BAR_OFFSET - (BN_MAX / 2 + 4) * 4);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t smem_base = smem_u32(smem);
   const uint32_t bar_base = smem_u32(bars);
-  // full[s] = bar_base + 8s, empty[s] = bar_base + 8(STAGES + s), accumulator = 8(2 STAGES)
+  // full[s] = bar_base + 8s, empty[s] = bar_base + 8(STAGES + s), accumulator = 8(2 STAGES),
+  // (TMEM slot, abort flag), split-K reduction copies = 8(2 STAGES + 2)
   const uint32_t acc_bar = bar_base + 8 * (2 * STAGES);
+  const uint32_t red_bar = bar_base + 8 * (2 * STAGES + 2);
 
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -112,6 +185,7 @@ __global__ void __launch_bounds__(128, 1)
       mbar_init(bar_base + 8 * (STAGES + s), 1);
     }
     mbar_init(acc_bar, 1);
+    mbar_init(red_bar, 1);
     fence_mbar_init();
     tma_prefetch_desc(&tm_w);
     tma_prefetch_desc(&tm_x);
@@ -162,7 +236,7 @@ __global__ void __launch_bounds__(128, 1)
 
   uint32_t p_stage = 0, p_phase = 0;  // producer ring position
   uint32_t c_stage = 0, c_phase = 0;  // MMA ring position
-  uint32_t acc_phase = 0;
+  uint32_t acc_phase = 0, red_phase = 0;
 
   for (int tile = cl_id; tile < tiles; tile += n_cl) {
     const int ft = tile % n_ft, tt = tile / n_ft;
@@ -171,6 +245,12 @@ __global__ void __launch_bounds__(128, 1)
     const int n_mma = (rows + 15) & ~15;
     const int nbox = (n_mma + XBOX - 1) / XBOX;
     bool ok = *sh_abort == 0;
+    // The epilogue's bias values, loaded now so that their latency hides under the main
+    // loop: the direct drain takes feature ft*BM + tid, the split-K reduction features
+    // ft*BM + 4*lane .. +3 (a thread's items all share its lane).
+    const float bias1 = ft * BM + tid < a.n_out ? __ldg(a.epi.bias + ft * BM + tid) : 0.f;
+    const float4 bias4 = ft * BM + 4 * lane < a.n_out ? __ldg(reinterpret_cast<const float4*>(a.epi.bias + ft * BM) + lane)
+                                                      : make_float4(0.f, 0.f, 0.f, 0.f);
 
     if (ok && has_k) {
       if (warp == 0) {
@@ -244,11 +324,7 @@ __global__ void __launch_bounds__(128, 1)
         for (int c0 = 0; c0 < rows; c0 += 16) {
           float v[16];
           tmem_ld16(trow + c0, v);
-          if (f < a.n_out) {
-#pragma unroll
-            for (int j = 0; j < 16; ++j)
-              if (c0 + j < rows) epilogue_store(a.epi, row0 + c0 + j, f, v[j]);
-          }
+          if (f < a.n_out) epilogue_column16(a.epi, row0 + c0, min(16, rows - c0), f, bias1, v);
         }
       }
     } else {
@@ -260,12 +336,14 @@ __global__ void __launch_bounds__(128, 1)
       const int slot = a.defer ? tile * csize + crank : cl_id * csize + crank;
       float* mine = a.partials + static_cast<size_t>(slot) * BN_MAX * BM;
       if (ok && has_k) {
-        for (int c0 = 0; c0 < rows; c0 += 16) {
-          float v[16];
-          tmem_ld16(trow + c0, v);
+        // 32 accumulator columns per TMEM load (columns past n_mma are allocated, unused)
+        for (int c0 = 0; c0 < rows; c0 += 32) {
+          uint32_t v[32];
+          tmem_ld32_async(trow + c0, v);
+          tmem_ld_wait_regs(v);
 #pragma unroll
-          for (int j = 0; j < 16; ++j)
-            if (c0 + j < rows) mine[(c0 + j) * BM + fl] = v[j];
+          for (int j = 0; j < 32; ++j)
+            if (c0 + j < rows) mine[(c0 + j) * BM + fl] = __uint_as_float(v[j]);
         }
       } else {
         for (int c = 0; c < rows; ++c) mine[c * BM + fl] = 0.f;
@@ -276,29 +354,47 @@ __global__ void __launch_bounds__(128, 1)
         continue;
       }
       cluster_sync();  // every partial of this tile is in the scratch
-      if (ok) {
-        const int c_lo = crank * rows / csize, c_hi = (crank + 1) * rows / csize;
-        const int f4 = ft * BM + 4 * lane;
-        const float* slots = a.partials + static_cast<size_t>(cl_id * csize) * BN_MAX * BM;
-        for (int c = c_lo + warp; c < c_hi; c += 4) {
-          float4 p[MAX_CLUSTER];
-#pragma unroll
-          for (int s = 0; s < MAX_CLUSTER; ++s)
-            if (s < csize)
-              p[s] = __ldcg(reinterpret_cast<const float4*>(slots + (static_cast<size_t>(s) * BN_MAX + c) * BM + 4 * lane));
-          float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-          for (int s = 0; s < MAX_CLUSTER; ++s)
-            if (s < csize) {
-              acc.x += p[s].x;
-              acc.y += p[s].y;
-              acc.z += p[s].z;
-              acc.w += p[s].w;
+      const int c_lo = crank * rows / csize, c_hi = (crank + 1) * rows / csize, nr = c_hi - c_lo;
+      if (ok && nr > 0) {
+        // This CTA's rows of every slot come into the (idle) stage memory with one bulk
+        // copy per slot, so the reduction costs one round trip to L2 however many rows
+        // it covers; then slots are summed in rank order (deterministic).
+        float* red = reinterpret_cast<float*>(smem);  // [csize][nr][BM]
+        const bool need_tok = epi_needs_tok(a.epi.kind);
+        if (tid == 0) {
+          fence_proxy_async_global();  // the peers' generic stores, acquired above, before the copies
+          mbar_arrive_expect_tx(red_bar, static_cast<uint32_t>(csize * nr * BM * 4));
+          for (int s = 0; s < csize; ++s)
+            bulk_load(smem_base + static_cast<uint32_t>(s * nr * BM * 4),
+                      a.partials + (static_cast<size_t>(cl_id * csize + s) * BN_MAX + c_lo) * BM,
+                      static_cast<uint32_t>(nr * BM * 4), red_bar);
+        }
+        if (need_tok && tid < nr) red_tok[tid] = __ldcg(a.epi.rowtok + row0 + c_lo + tid);
+        __syncthreads();
+        if (!mbar_wait(red_bar, red_phase)) {
+          atomicExch(a.err, kErrWaitTmaFull);
+          *sh_abort = 1;
+        }
+        red_phase ^= 1;
+        if (*sh_abort == 0) {
+          const float4* r4 = reinterpret_cast<const float4*>(red);
+          for (int e = tid; e < nr * (BM / 4); e += 128) {
+            const int c = e / (BM / 4), q = e % (BM / 4), f4 = ft * BM + 4 * q;
+            if (f4 >= a.n_out) continue;
+            float4 acc = r4[c * (BM / 4) + q];
+            for (int s = 1; s < csize; ++s) {
+              const float4 p = r4[(s * nr + c) * (BM / 4) + q];
+              acc.x += p.x;
+              acc.y += p.y;
+              acc.z += p.z;
+              acc.w += p.w;
             }
-          const float vals[4] = {acc.x, acc.y, acc.z, acc.w};
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-            if (f4 + j < a.n_out) epilogue_store(a.epi, row0 + c, f4 + j, vals[j]);
+            float4 old = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (a.epi.kind == kEpiResid)
+              old = __ldcg(reinterpret_cast<const float4*>(a.epi.out_f32 +
+                                                           static_cast<size_t>(row0 + c_lo + c) * a.epi.ld_out + f4));
+            epilogue_store4(a.epi, row0 + c_lo + c, f4, acc, bias4, need_tok ? red_tok[c] : 0, old);
+          }
         }
       }
       if (tile + n_cl < tiles) cluster_sync();  // the next tile rewrites the slots
@@ -465,24 +561,21 @@ __global__ void __launch_bounds__(WS_THREADS, 1)
       const int ft = tile % n_ft, tt = tile / n_ft;
       const int row0 = tt * BN_MAX, rows = min(BN_MAX, M - row0);
       const int b = iter & 1;
+      const int f = ft * BM + quarter * 32 + lane;
+      const float bias_f = f < a.n_out ? __ldg(a.epi.bias + f) : 0.f;  // loads while the MMAs run
       if (!mbar_wait(accf + 8 * b, (iter >> 1) & 1)) {
         atomicExch(a.err, kErrWaitAccum);
         *sh_abort = 1;
         break;
       }
       tc_fence_after();
-      const int f = ft * BM + quarter * 32 + lane;
       const uint32_t acc = trow + static_cast<uint32_t>(b * BN_MAX);
       const int hrows = ((rows + 31) / 32) * 16;
       const int r_lo = half * hrows, r_hi = min(rows, r_lo + hrows);
       for (int c0 = r_lo; c0 < r_hi; c0 += 16) {
         float v[16];
         tmem_ld16(acc + c0, v);
-        if (f < a.n_out) {
-#pragma unroll
-          for (int j = 0; j < 16; ++j)
-            if (c0 + j < r_hi) epilogue_store(a.epi, row0 + c0 + j, f, v[j]);
-        }
+        if (f < a.n_out) epilogue_column16(a.epi, row0 + c0, min(16, r_hi - c0), f, bias_f, v);
       }
       tc_fence_before();
       __syncwarp();
