@@ -49,6 +49,7 @@ constexpr int AQ = 128;            // queries per item (MMA M)
 constexpr int AKMAX = 256;         // max keys per CTA (MMA N of S)
 constexpr int KROWS = 64;          // rows of one K/V TMA box
 constexpr int SLICE_Q = AQ * 128;  // [128 rows][128 B]: 16 KB (a Q slice or a 64-key P slice)
+constexpr int QBOX = 32;           // rows of one query TMA box
 constexpr int MAX_SPLITS = 8;
 
 // Shared-memory and TMEM layout of one CTA for kpc keys and head width dhp (padded to
@@ -251,9 +252,13 @@ __global__ void __launch_bounds__(NT, 1)
     const bool patch = first && pre;
     first = false;
     if (tid == 0) {
-      mbar_arrive_expect_tx(bq, NSL * SLICE_Q);
+      // only the 32-row boxes that hold the item's queries (rows past them are never stored)
+      const int nqb = (it.nq + QBOX - 1) / QBOX;
+      mbar_arrive_expect_tx(bq, static_cast<uint32_t>(NSL * nqb * QBOX * 128));
       for (int sl = 0; sl < NSL; ++sl)
-        tma_load_2d(sb + L.off_q + sl * SLICE_Q, &tm_q, it.h * dh + sl * 64, it.r0, bq, pol_q);
+        for (int b = 0; b < nqb; ++b)
+          tma_load_2d(sb + L.off_q + sl * SLICE_Q + b * QBOX * 128, &tm_q, it.h * dh + sl * 64, it.r0 + b * QBOX, bq,
+                      pol_q);
       if (!patch && ngroups > 0) {
         load_kv(bk, L.off_k, &tm_k, it.v, it.h, 0);
         load_kv(bv, L.off_v, &tm_v, it.v, it.h, 0);

@@ -43,6 +43,7 @@ struct TimelineSlot {
 struct GemmPlan {
   int bn = 64, csize = 1, n_clusters = 1;
   bool defer = false;  // residual GEMMs: leave the split partials to the next layer norm
+  bool vsplit = false; // deferred: K split over CTAs launched without clusters
 };
 
 enum GemmSlot { kGemmEmbed = 0, kGemmQKV, kGemmO, kGemmUp, kGemmDown, kGemmSlots };
@@ -129,7 +130,7 @@ struct ivit_handle {
   float *b_pe = nullptr, *pos = nullptr, *lnfg = nullptr, *lnfb = nullptr;
   std::vector<LayerW> layers;
   CUtensorMap tm_pe, tm_patches, tm_xn, tm_o, tm_h;
-  CUtensorMap tm_qa;     // packed queries, 64 x 128 boxes, 128-byte swizzle (tcgen05 attention)
+  CUtensorMap tm_qa;     // packed queries, 64 x 32 boxes, 128-byte swizzle (tcgen05 attention)
   bool attn_tc = true;   // tensor-core attention (IVIT_ATTN=simt selects the SIMT kernel)
   int attn_splits_full = 1, attn_splits_inc = 1;  // key splits (CTAs per item) of that kernel
 
@@ -553,33 +554,70 @@ int setup(ivit_handle* h, const uint16_t* wb) {
       h->plan_inc[g] = g == kGemmEmbed ? h->plan_full[g]
                                        : plan_gemm(h->num_sms, bn_inc, shapes[g][0], shapes[g][1], m_inc);
       h->plan_band[0][g] = h->plan_inc[g];
+      // (the band of all rows runs the full encode's plans: it attends like one too)
       for (int b = 1; b < h->n_bands; ++b)
-        h->plan_band[b][g] = g == kGemmEmbed ? h->plan_full[g]
-                                             : plan_gemm(h->num_sms, h->band_ub[b] <= 64 ? 64 : 256, shapes[g][0],
-                                                         shapes[g][1], h->band_ub[b]);
+        h->plan_band[b][g] = g == kGemmEmbed || h->band_ub[b] >= static_cast<int>(M)
+                                 ? h->plan_full[g]
+                                 : plan_gemm(h->num_sms, h->band_ub[b] <= 256 ? 64 : 256, shapes[g][0], shapes[g][1],
+                                             h->band_ub[b]);
     }
     // Residual GEMMs split over clusters leave their partials to the layer norm that
     // follows (one slot per tile and split, sized for the most rows the plan can see),
     // while that scratch stays under 64 MB.
+    // A deferred residual GEMM needs no cluster barrier, so its K split runs over plain
+    // CTAs: the split is chosen by the same cost model without the cluster packing limit,
+    // as many splits as fill the SMs once (at most 16, the layer norm's limit).
+    auto replan_free = [&](GemmPlan& pl, int n_out, int k, int m_expected) {
+      const int n_ft = (n_out + 127) / 128, n_tt = (m_expected + pl.bn - 1) / pl.bn, n_kb = (k + 63) / 64;
+      const int tiles = std::max(1, n_ft * n_tt);
+      double best_cost = 1e30;
+      GemmPlan best = pl;
+      for (int c = 2; c <= std::min(16, n_kb); ++c) {
+        const int rounds = (tiles * c + h->num_sms - 1) / h->num_sms;
+        const double cost = rounds * (4.0 + 0.35 * ((n_kb + c - 1) / c));
+        if (cost < best_cost - 1e-9) {
+          best_cost = cost;
+          best.csize = c;
+          best.n_clusters = tiles;
+        }
+      }
+      if (best_cost < 1e29 && !std::getenv("IVIT_NO_VSPLIT")) {
+        pl = best;
+        pl.vsplit = true;
+      }
+    };
     auto set_defer = [&](GemmPlan& pl, int n_out, int m_bound) {
       const size_t slots = static_cast<size_t>((n_out + 127) / 128) * ((m_bound + pl.bn - 1) / pl.bn) * pl.csize;
       pl.defer = pl.csize > 1 && !std::getenv("IVIT_NO_DEFER") && slots * pl.bn * 128 * 4 <= (64ull << 20) &&
                  h->D % 4 == 0 && h->D <= 4096;
     };
+    // a deferred plan re-planned without clusters, kept if its scratch still fits
+    auto refine = [&](GemmPlan& pl, int g, int m_expected, int m_bound) {
+      if (!pl.defer) return;
+      const GemmPlan orig = pl;
+      replan_free(pl, shapes[g][0], shapes[g][1], m_expected);
+      set_defer(pl, static_cast<int>(D), m_bound);
+      if (!pl.defer) pl = orig;
+    };
     for (int g : {static_cast<int>(kGemmO), static_cast<int>(kGemmDown)}) {
       set_defer(h->plan_full[g], static_cast<int>(D), static_cast<int>(M));
       set_defer(h->plan_inc[g], static_cast<int>(D), static_cast<int>(M));
+      refine(h->plan_full[g], g, static_cast<int>(M), static_cast<int>(M));
+      refine(h->plan_inc[g], g, std::max(1, static_cast<int>(M / 10)), static_cast<int>(M));
       h->plan_band[0][g] = h->plan_inc[g];
-      for (int b = 1; b < h->n_bands; ++b) set_defer(h->plan_band[b][g], static_cast<int>(D), h->band_ub[b]);
+      for (int b = 1; b < h->n_bands; ++b) {
+        set_defer(h->plan_band[b][g], static_cast<int>(D), h->band_ub[b]);
+        refine(h->plan_band[b][g], g, h->band_ub[b], h->band_ub[b]);
+      }
     }
     if (std::getenv("IVIT_DEBUG")) {
       static const char* names[kGemmSlots] = {"embed", "qkv", "out", "up", "down"};
       for (int g = 0; g < kGemmSlots; ++g)
-        std::fprintf(stderr, "ivit gemm %-5s full bn=%d cluster=%d x %d (fit %d) | inc bn=%d cluster=%d x %d (fit %d)\n",
-                     names[g], h->plan_full[g].bn, h->plan_full[g].csize, h->plan_full[g].n_clusters,
-                     ivit::gemm_max_clusters(h->plan_full[g].bn, h->plan_full[g].csize), h->plan_inc[g].bn,
-                     h->plan_inc[g].csize, h->plan_inc[g].n_clusters,
-                     ivit::gemm_max_clusters(h->plan_inc[g].bn, h->plan_inc[g].csize));
+        std::fprintf(stderr, "ivit gemm %-5s full bn=%d %s=%d x %d (fit %d) | inc bn=%d %s=%d x %d (fit %d)\n",
+                     names[g], h->plan_full[g].bn, h->plan_full[g].vsplit ? "split" : "cluster", h->plan_full[g].csize,
+                     h->plan_full[g].n_clusters, ivit::gemm_max_clusters(h->plan_full[g].bn, h->plan_full[g].csize),
+                     h->plan_inc[g].bn, h->plan_inc[g].vsplit ? "split" : "cluster", h->plan_inc[g].csize,
+                     h->plan_inc[g].n_clusters, ivit::gemm_max_clusters(h->plan_inc[g].bn, h->plan_inc[g].csize));
       for (int b = 1; b < h->n_bands; ++b)
         std::fprintf(stderr, "ivit band %d (<= %d rows): attention splits %d\n", b, h->band_ub[b], h->attn_splits_band[b]);
     }
@@ -744,7 +782,7 @@ int setup(ivit_handle* h, const uint16_t* wb) {
   if (!make_map(&h->tm_patches, h->patches, h->KPAD, M, h->KPAD * 2, 64, 32) ||
       !make_map(&h->tm_xn, h->xn, D, M, D * 2, 64, 32) ||
       !make_map(&h->tm_o, h->o, D, M, D * 2, 64, 32) ||
-      !make_map(&h->tm_qa, h->q, D, M, D * 2, 64, 128) ||
+      !make_map(&h->tm_qa, h->q, D, M, D * 2, 64, 32) ||
       !make_map(&h->tm_h, h->hbuf, F, M, F * 2, 64, 32))
     return h->fail(IVIT_ERR_CUDA, "cuTensorMapEncodeTiled failed for an activation buffer");
   if (int r = setup_persistent(h)) return r;
@@ -1035,6 +1073,7 @@ int run_layers(ivit_handle* h, const GemmPlan* plan, int attn_splits, bool full,
     a.epi.out_f32 = h->x;
     a.epi.ld_out = D;
     a.defer = pl.defer ? 1 : 0;
+    a.vsplit = pl.defer && pl.vsplit ? pl.csize : 0;
     if (int r = gemm(h, pl, tw, tx, a, s)) return r;
     if (pl.defer) {
       pend.partials = h->gemm_partials;

@@ -200,8 +200,9 @@ __global__ void __launch_bounds__(128, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  const int csize = static_cast<int>(cluster_nctarank());
-  const int crank = static_cast<int>(cluster_ctarank());
+  // a deferred launch may split K over consecutive CTAs without clusters (a.vsplit)
+  const int csize = a.vsplit > 0 ? a.vsplit : static_cast<int>(cluster_nctarank());
+  const int crank = a.vsplit > 0 ? static_cast<int>(blockIdx.x) % a.vsplit : static_cast<int>(cluster_ctarank());
   const int cl_id = blockIdx.x / csize, n_cl = gridDim.x / csize;
   // The row count comes from the selection kernel, at least two launches back: every
   // kernel of the library triggers its dependents only after its own wait, so that
@@ -597,7 +598,8 @@ cudaError_t launch_variant(const CUtensorMap& tm_w, const CUtensorMap& tm_x, con
   if (BN == 256 && csize == 1)
     return launch_ex(gemm_ws_kernel<BN>, dim3(n_clusters), dim3(WS_THREADS), GemmSmem<BN>::TOTAL, s, 1, tm_w, tm_x,
                      a);
-  // cluster dims are always given (also for a single CTA) so %cluster_nctarank is exact
+  // cluster dims are always given (also for a single CTA) so %cluster_nctarank is exact;
+  // a launch with a virtual split (deferred partials, no cluster barrier) runs clusters of one
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(n_clusters * csize);
   cfg.blockDim = dim3(128);
@@ -605,7 +607,7 @@ cudaError_t launch_variant(const CUtensorMap& tm_w, const CUtensorMap& tm_x, con
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = csize;
+  attr[0].val.clusterDim.x = a.vsplit > 0 ? 1 : csize;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;

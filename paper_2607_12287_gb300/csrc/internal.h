@@ -88,6 +88,10 @@ struct GemmArgs {
   // (layernorm_sum, for the residual epilogue).  The scratch then holds
   // n_ft * ceil(M / BN_MAX) * csize slots.
   int defer = 0;
+  // With defer set and vsplit > 0, K is split over vsplit consecutive CTAs launched as
+  // clusters of one (no cluster barrier is needed to leave the partials): the split
+  // count is then free of the GPC packing that limits cluster sizes.
+  int vsplit = 0;
   unsigned long long* stamp = nullptr;  // timeline stamps of this launch (or null)
   GemmEpilogue epi;
 };
@@ -285,7 +289,7 @@ size_t attention_tc_smem(int n_tok, int dh, int key_splits);
 
 // O[r] = softmax(Q[r] K_v^T / sqrt(dh)) V_v per head on the tensor cores, for the packed
 // query rows r of each view v, over the N cached keys/values of that view.  tm_q: the
-// packed queries bf16 [rows][D] with box 64 columns x 128 rows; tm_k / tm_v: this
+// packed queries bf16 [rows][D] with box 64 columns x 32 rows; tm_k / tm_v: this
 // layer's caches bf16 [SV*N][D] with box 64 columns x attention_tc_kv_box_rows(); all
 // three with 128-byte swizzle.  Grid: clusters of
 // key_splits CTAs (128 threads each), at most max_ctas CTAs, walking the (query tile,
