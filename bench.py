@@ -60,8 +60,9 @@ def read_peaks() -> dict:
     if os.path.exists(p):
         with open(p) as f:
             d = json.load(f)
-        return {"hbm_gbs": d.get("hbm_gbs"), "bf16_tflops": d.get("bf16_tflops"), "source": "measured"}
-    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
+        return {"hbm_gbs": d.get("hbm_gbs"), "bf16_tflops": d.get("bf16_tflops"),
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained") or d.get("bf16_tflops"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
 
 
 L2_BYTES = 129e6  # GB300 L2
@@ -87,6 +88,28 @@ def algorithmic_bytes_per_step(wl, rows_per_step: float) -> float:
     embed = 3 * 4.0 * sv * N * D
     writes = rows_per_step * (2 * 2 * L * D + 2 * D)
     return weight_matrix_bytes(s) + kv + frames + embed + writes
+
+
+def ideal_ms_per_step(wl, rows_per_step: float, full: bool, peaks: dict) -> dict:
+    """Roofline time of one call: the larger of its algorithmic bytes at the measured HBM
+    copy bandwidth and its FLOPs at the measured sustained bf16 tensor throughput.  A
+    full encode runs every block on all SV*N tokens and writes every cached K/V; an
+    incremental call runs them on ``rows_per_step`` updated tokens and reads every cached
+    K/V (Sec. III-B, Eq. 4-5).  Both stream the weights once and embed every patch."""
+    s = wl.shape
+    N, D, F, L, sv = s.n_tokens, s.dim, s.mlp_dim, s.depth, wl.sv
+    kp = s.patch * s.patch * 3
+    rows = float(sv * N) if full else float(rows_per_step)
+    flops = 2.0 * sv * N * D * kp + L * (rows * 2.0 * (4 * D * D + 2 * D * F) + 4.0 * rows * N * D)
+    kv_all = 2.0 * 2 * L * sv * N * D
+    if full:
+        byts = weight_matrix_bytes(s) + kv_all + sv * s.img_h * s.img_w * 3 + 3 * 4.0 * sv * N * D
+    else:
+        byts = algorithmic_bytes_per_step(wl, rows)
+    t_mem = byts / (peaks["hbm_gbs"] * 1e9)
+    t_mma = flops / (peaks["bf16_tflops_sustained"] * 1e12)
+    return {"ms": 1e3 * max(t_mem, t_mma), "bound": "hbm" if t_mem >= t_mma else "tensor", "bytes": byts,
+            "flops": flops}
 
 
 def gemm_traffic_ratio():
@@ -441,6 +464,8 @@ def main() -> None:
     traffic = ratio * gemm_bytes_step / gemm_launches if (ratio is not None and gemm_launches) else None
     rows_step = float(changed.mean())
     call_bytes = algorithmic_bytes_per_step(wl, rows_step)
+    ideal_inc = ideal_ms_per_step(wl, rows_step, False, peaks)
+    ideal_full = ideal_ms_per_step(wl, rows_step, True, peaks)
     wbytes = weight_matrix_bytes(wl.shape)
     line = {
         "metric": METRIC, "value": value, "unit": "frames/s", "n_gpus": world, "steps": args.steps,
@@ -461,6 +486,12 @@ def main() -> None:
         "full_encode_ms_per_step": full_ms / args.steps,
         "full_encode_frames_per_s": frames_total / (full_ms / 1e3),
         "speedup_vs_full": full_ms / inc_ms,
+        # the same ratio at the roofline (measured peaks): what a perfect implementation of
+        # both calls would show on this workload
+        "ideal_speedup_vs_full": ideal_full["ms"] / ideal_inc["ms"],
+        "ideal_ms_per_step": {"incremental": ideal_inc, "full": ideal_full,
+                              "frac_incremental": ideal_inc["ms"] / ms_step,
+                              "frac_full": ideal_full["ms"] / (full_ms / args.steps)},
         "odd_even_ms_per_step": oe_ms / args.steps,  # Sec. III-B alternating full / incremental calls
         "quality_vs_full": quality_default,
         "mlp_all_tokens": mlp_all,

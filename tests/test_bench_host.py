@@ -77,3 +77,25 @@ def test_algorithmic_bytes_per_step_so400m():
     b = bench.algorithmic_bytes_per_step(wl, 26)
     assert 0.85e9 < b < 0.87e9
     assert bench.algorithmic_bytes_per_step(wl, 52) > b
+
+
+def test_ideal_speedup_follows_the_roofline():
+    # One 224 px So400m view: both calls stream the same 824 MB of weights and the full
+    # encode's 220 GFLOP take as long at the tensor peak, so a perfect implementation
+    # gains nothing from skipping rows (ratio ~1).  Three views with 5/15/30% updated rows
+    # share the weights across three views' worth of full-encode FLOPs: about 2.7.
+    pk = {"hbm_gbs": 6785.5, "bf16_tflops_sustained": 1716.2}
+    one = synth.WORKLOADS["so400m_224_1view"]
+    inc = bench.ideal_ms_per_step(one, 0.1 * 256, False, pk)
+    full = bench.ideal_ms_per_step(one, 0.1 * 256, True, pk)
+    assert inc["bound"] == "hbm" and full["bound"] == "tensor"
+    assert 0.95 < full["ms"] / inc["ms"] < 1.05
+    # the full encode's FLOPs: 2 * params-per-token * tokens plus attention, per layer
+    s = one.shape
+    per_row = 2.0 * (4 * s.dim * s.dim + 2 * s.dim * s.mlp_dim) + 4.0 * s.n_tokens * s.dim
+    embed = 2.0 * s.n_tokens * s.dim * s.patch * s.patch * 3
+    assert abs(full["flops"] - (embed + s.depth * s.n_tokens * per_row)) < 1e-6 * full["flops"]
+    three = synth.WORKLOADS["so400m_224_3view"]
+    rows = 256 * (0.05 + 0.15 + 0.30)
+    r3 = bench.ideal_ms_per_step(three, rows, True, pk)["ms"] / bench.ideal_ms_per_step(three, rows, False, pk)["ms"]
+    assert 2.5 < r3 < 2.9
