@@ -408,16 +408,19 @@ __global__ void __launch_bounds__(NT, 1)
       ++ph_g;
       if (tid == 0 && g + 1 < ngroups) load_kv(bv, L.off_v, &tm_v, it.v, it.h, g + 1);  // V tile consumed
       if (wrow) {  // warp-uniform: tcgen05.ld is a warp-collective instruction
+        // two chunks' loads in flight per wait (one for the widest heads with two threads
+        // per row, whose registers are otherwise spent)
+        constexpr int OB = (DHP >= 112 && NH > 1) ? 1 : 2;
 #pragma unroll
-        for (int q = 0; q < OCH; q += 2) {  // two chunks' loads in flight per wait
-          uint32_t ov[2][16];
+        for (int q = 0; q < OCH; q += OB) {
+          uint32_t ov[OB][16];
 #pragma unroll
-          for (int t = 0; t < 2; ++t)
+          for (int t = 0; t < OB; ++t)
             if (q + t < OCH && (hf + (q + t) * NH) * 16 < DHP)
               tmem_ld16_async(trow + L.tm_o + (hf + (q + t) * NH) * 16, ov[t]);
           tmem_ld_wait();
 #pragma unroll
-          for (int t = 0; t < 2; ++t) {
+          for (int t = 0; t < OB; ++t) {
             tmem_regs_after_wait16(ov[t]);
             if (q + t < OCH && (hf + (q + t) * NH) * 16 < DHP) {
 #pragma unroll
