@@ -561,12 +561,11 @@ int setup(ivit_handle* h, const uint16_t* wb) {
                                  : plan_gemm(h->num_sms, h->band_ub[b] <= 256 ? 64 : 256, shapes[g][0], shapes[g][1],
                                              h->band_ub[b]);
     }
-    // Residual GEMMs split over clusters leave their partials to the layer norm that
-    // follows (one slot per tile and split, sized for the most rows the plan can see),
-    // while that scratch stays under 64 MB.
-    // A deferred residual GEMM needs no cluster barrier, so its K split runs over plain
-    // CTAs: the split is chosen by the same cost model without the cluster packing limit,
-    // as many splits as fill the SMs once (at most 16, the layer norm's limit).
+    // Residual GEMMs with a K split leave their partials to the layer norm that follows
+    // (one slot per tile and split, sized for the most rows the plan can see), while that
+    // scratch stays under 64 MB.  Needing no cluster barrier, such a GEMM then splits K
+    // over plain CTAs, with the split re-chosen by the same cost model without the
+    // cluster packing limit (at most 16 splits, the layer norm's limit).
     auto replan_free = [&](GemmPlan& pl, int n_out, int k, int m_expected) {
       const int n_ft = (n_out + 127) / 128, n_tt = (m_expected + pl.bn - 1) / pl.bn, n_kb = (k + 63) / 64;
       const int tiles = std::max(1, n_ft * n_tt);

@@ -104,12 +104,14 @@ __device__ __forceinline__ void epilogue_column16(const GemmEpilogue& e, int r0,
                                                   const float (&v)[16]) {
   int tok[16];
   float old[16];
+  // (the QKV epilogue's queries stay in packed rows: only its keys and values need tokens)
+  const bool need_tok = e.kind == kEpiScatterF32 || (e.kind == kEpiQKV && f >= e.dim);
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
     tok[j] = 0;
     old[j] = 0.f;
     if (j < n) {
-      if (epi_needs_tok(e.kind)) tok[j] = __ldcg(e.rowtok + r0 + j);
+      if (need_tok) tok[j] = __ldcg(e.rowtok + r0 + j);
       if (e.kind == kEpiResid) old[j] = __ldcg(e.out_f32 + static_cast<size_t>(r0 + j) * e.ld_out + f);
     }
   }
