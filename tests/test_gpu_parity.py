@@ -322,3 +322,14 @@ def test_timeline_records_every_launch(pkg):
             enc.close()
     for a, b in zip(*outs):
         assert torch.equal(a, b)
+
+
+def test_maximum_view_count(pkg, oracle_mod):
+    # 4096 views, the most a handle takes (1024 streams x 4 views of a 4-token encoder):
+    # one selection CTA per view, the cold-view mask and the packed-row offsets at their
+    # largest, 16384 rows through 256-row GEMM tiles and 4096 attention items
+    shape = synth.EncoderShape(16, 16, 8, 64, 1, 1, 128, synth.GELU_TANH)
+    w = synth.make_weights(shape, 171)
+    frames = list(synth.stream_random(shape, 4096, 3, 172, change_p=0.3))
+    stats = run_side_by_side(pkg, oracle_mod, shape, w, frames, 1024, 4, check_caches=True)
+    assert all(0 < int(st[2].sum()) < 4096 * shape.n_tokens for st in stats[1:])
